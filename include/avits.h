@@ -1,0 +1,232 @@
+/*
+ * avits.h — C ABI of the AViTS resolution-transition hot path on GB300 (sm_103a).
+ *
+ * AViTS (Adaptive Spatiotemporal Token Selection, arxiv 2608.17995) runs a
+ * diffusion transformer at half resolution, scores every low-resolution image
+ * token by how strongly it attends to the text (spatial importance, Sec. 3.3.1,
+ * Eq. 3-5) and by how much it moves between denoising steps (temporal
+ * importance, Sec. 3.3.2), fuses the two min-max normalised scores (Eq. 8),
+ * keeps the top-K tokens (Eq. 9) and upsamples only those (Sec. 3.2, Stage 2).
+ * After Stage 2 the remaining tokens are expanded and the sequence is put back
+ * in spatial order (Sec. 3.2, Stage 3).  This library computes that transition:
+ *
+ *   avits_score_spatial       Eq. 3 + Eq. 5   per-token text attention mass
+ *   avits_score_temporal      Sec. 3.3.2      per-token relative step change
+ *   avits_fuse_select         Sec. 3.3.3, Eq. 8 + Eq. 9   min-max, fuse, top-K
+ *   avits_selective_upsample  Sec. 3.2 Stage 2   packed mixed-resolution sequence
+ *   avits_merge_final         Sec. 3.2 Stage 3   dense full-resolution latent
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - Every tensor pointer is DEVICE memory owned by the caller.  The library
+ *    allocates no device memory; the split-key partial sums of
+ *    avits_score_spatial and the cell map of bilinear avits_merge_final live
+ *    in a caller workspace whose size a *_workspace() query returns.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream).  Every call is asynchronous and stream ordered; none
+ *    synchronises the host except avits_device_status().
+ *  - Arguments are checked on the host before anything is launched.  A bad
+ *    argument returns AVITS_ERR_INVALID_ARG (or AVITS_ERR_UNSUPPORTED for a
+ *    combination the kernels do not implement) and launches nothing.
+ *  - A failed launch returns AVITS_ERR_CUDA (the CUDA error is cleared and
+ *    its text kept for avits_last_error_string()).
+ *  - Errors found on the device (a bounded wait that ran out, a NaN score, a
+ *    mixed sequence that does not tile the output frame) are OR-ed into a
+ *    per-device status word, read and cleared by avits_device_status().
+ *  - Dtypes: AVITS_BF16 (bfloat16 inputs, fp32 arithmetic) and AVITS_F32.
+ *    Scores are always fp32.
+ *  - Latent tokens hold C*p*p values ordered (channel, patch-row, patch-col),
+ *    p = 2 (the 2x2 patchification of FLUX-family models).
+ *  - Token grids are raster ordered: token i of a gh x gw grid sits at row
+ *    i / gw, column i % gw.
+ */
+#ifndef AVITS_H
+#define AVITS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  AVITS_OK = 0,
+  AVITS_ERR_INVALID_ARG = 1,
+  AVITS_ERR_UNSUPPORTED = 2,
+  AVITS_ERR_CUDA = 3,
+  AVITS_ERR_TIMEOUT = 4,   /* device: a bounded wait gave up */
+  AVITS_ERR_NAN = 5,       /* device: a NaN reached the fused score */
+  AVITS_ERR_COVERAGE = 6   /* device: merge input does not tile the frame */
+} avits_status;
+
+typedef enum { AVITS_F32 = 0, AVITS_BF16 = 1 } avits_dtype;
+
+typedef enum { AVITS_UP_NEAREST = 0, AVITS_UP_BILINEAR = 1 } avits_upmode;
+
+/* ------------------------------------------------------------------------
+ * Spatial importance, Sec. 3.3.1, Eq. 3 with the joint-attention extraction
+ * of Eq. 4-5.  For batch b, head h and image query i:
+ *
+ *     l_ij  = softmax_scale * <q_bhi, k_bhj>                 j = 0 .. Nk-1
+ *     mass  = sum_{j<L} exp(l_ij) / sum_{j<Nk} exp(l_ij)     (text keys first)
+ *     A[b,i] = (accumulate ? A[b,i] : 0) + weight * (1/H) * sum_h mass
+ *
+ * i.e. the softmax over ALL keys (text, image and, for editing models, the
+ * reference-image keys) restricted to the L text columns and summed, then
+ * averaged over heads (Eq. 3).  The score matrix is never materialised.
+ * `accumulate` + `weight` aggregate over the selected blocks and the N_T
+ * collection steps (end of Sec. 3.3.1): e.g. weight = 1/(blocks*N_T).
+ *
+ * q_img : [B,H,M,d] image-query projections after the model's QK norm (and
+ *         RoPE if the model applies it before attention).  Element strides
+ *         q_sb, q_sh, q_sn; the d axis is contiguous.  May be a strided view
+ *         of the joint Q of Eq. 4 (skip the L text rows).
+ * k_all : [B,H,Nk,d] joint keys, the L text keys FIRST, then the image keys,
+ *         then optional reference keys.  Strides k_sb, k_sh, k_sn; d contiguous.
+ * dt    : AVITS_BF16 (tensor-core path, needs d in {64,128}, 16-byte aligned
+ *         base and strides) or AVITS_F32 (CUDA-core path, any d <= 256).
+ * softmax_scale > 0 (1/sqrt(d) in the paper).  0 <= L <= Nk.
+ * A     : [B,M] fp32, written (accumulate = 0) or added to.
+ * lse_opt : NULL or [B,H,M,2] fp32 receiving (log sum_j exp l_ij over all
+ *         keys, the same over the text keys), natural log; -inf when a sum
+ *         underflows.
+ * workspace/ws_bytes : at least avits_score_spatial_workspace(...) bytes.
+ *         It MUST be zero-filled before its first use; every successful
+ *         call leaves it zero-filled again.  After a device error re-zero it.
+ *         One workspace must not be used by two calls running concurrently.
+ * ---------------------------------------------------------------------- */
+avits_status avits_score_spatial(const void* q_img, const void* k_all, avits_dtype dt,
+                                 int B, int H, int M, int Nk, int L, int d,
+                                 int64_t q_sb, int64_t q_sh, int64_t q_sn,
+                                 int64_t k_sb, int64_t k_sh, int64_t k_sn,
+                                 float softmax_scale, float weight, int accumulate,
+                                 float* A, float* lse_opt,
+                                 void* workspace, size_t ws_bytes, void* stream);
+
+/* Workspace bytes avits_score_spatial needs on the CURRENT device for these
+ * sizes (0 if it needs none).  Returns 0 as well for invalid sizes. */
+size_t avits_score_spatial_workspace(avits_dtype dt, int B, int H, int M, int Nk, int d);
+
+/* ------------------------------------------------------------------------
+ * Temporal importance.  Sec. 3.3.2 scores a token by how much its feature
+ * moves across the collected denoising steps.  This call takes the two most
+ * recent snapshots and returns the relative step change
+ *
+ *     V[b,i] = ||h_t[b,i,:] - h_prev[b,i,:]||_2 / (||h_prev[b,i,:]||_2 + eps)
+ *
+ * (eps = 1e-6 by default).  The paper's own N_T-snapshot step variance,
+ * Eq. 6-7, is avits_score_temporal_var below.
+ * h_t, h_prev : [B,N,D] contiguous, bf16 or fp32, 16-byte aligned.
+ * V : [B,N] fp32.  Sums of squares are accumulated in fp32.
+ * ---------------------------------------------------------------------- */
+avits_status avits_score_temporal(const void* h_t, const void* h_prev, avits_dtype dt,
+                                  int B, int N, int D, float eps, float* V, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Paper-form temporal importance, Sec. 3.3.2 Eq. 6-7: for each token the
+ * unbiased sample variance over N_T snapshots of every channel, averaged
+ * over the D channels.
+ * snaps : N_T pointers (a HOST array of device pointers), each to a [B,N,D]
+ *         contiguous snapshot, oldest first.  N_T >= 2.
+ * V : [B,N] fp32.  Two-pass (mean, then squared deviations) in fp32.
+ * ---------------------------------------------------------------------- */
+avits_status avits_score_temporal_var(const void* const* snaps, int n_t, avits_dtype dt,
+                                      int B, int N, int D, float* V, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Joint score and selection, Sec. 3.3.3, Eq. 8-9.  Per batch element:
+ *
+ *   A^ = (A - min A) / ((max A - min A) + eps_norm),   V^ likewise
+ *   S  = alpha * A^ + (1 - alpha) * V^                   (fp32, this op order)
+ *   sel = the k largest S; ties go to the LOWER token index (the paper breaks
+ *         ties with ~1e-6 Gaussian noise; this library is deterministic).
+ *         NaN ranks below every number; -0 and +0 are equal.
+ *
+ * A, V : [B,M] fp32.  0 <= k <= M, M <= 65536.
+ * S_opt : NULL or [B,M] fp32.
+ * sel_idx : [B,k] int32, the selected token indices in ascending order.
+ * sel_mask_opt : NULL or [B,M] uint8 (1 = selected).
+ * tok_offset : [B,M] int32, where token i starts in the mixed sequence:
+ *              i + 3 * (number of selected tokens before i).
+ * A NaN in S also sets AVITS_ERR_NAN in the device status word.
+ * ---------------------------------------------------------------------- */
+avits_status avits_fuse_select(const float* A, const float* V, int B, int M, float alpha,
+                               float eps_norm, int k, float* S_opt, int32_t* sel_idx,
+                               uint8_t* sel_mask_opt, int32_t* tok_offset, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Selective upsampling, Sec. 3.2 Stage 2: selected tokens are expanded to
+ * the next resolution, the others stay as they are, and all of them go into
+ * one packed mixed-resolution sequence of N_out = M + 3k tokens.
+ *
+ * Token i (input frame position (y,x), span s; without pos_in: (i/gw, i%gw),
+ * s = 1) is emitted at tok_offset[i]:
+ *   selected : 4 children c = 2a+b (a,b in {0,1}) at output positions
+ *              (2y + a*s, 2x + b*s), span s, each child = 2x upsample of
+ *              parent pixel (a,b): nearest broadcasts it; bilinear uses the
+ *              fixed weights 0.75/0.25 of a half-pixel-centred 2x resize with
+ *              edge clamping over the dense input latent.
+ *   deferred : the token unchanged at (2y, 2x), span 2s.
+ * Output positions are in the doubled frame (2gh x 2gw), usable directly as
+ * 2D RoPE ids.
+ *
+ * latent : [B,M,C*4] bf16/fp32.  Without pos_in, M = gh*gw (a dense grid).
+ * pos_in_opt/span_in_opt : NULL, or [B,M,2] / [B,M] int32 for a mixed input
+ *          (a second transition); nearest mode only.
+ * sel_mask, tok_offset : from avits_fuse_select.  k = number selected.
+ * out_latent : [B,M+3k,C*4] same dtype.  out_pos : [B,M+3k,2] (row, col).
+ * out_span : [B,M+3k].  out_src_tok : [B,M+3k] input token index.
+ * out_src_sub : [B,M+3k] int8, child number 0..3, or -1 for a deferred token.
+ * ---------------------------------------------------------------------- */
+avits_status avits_selective_upsample(const void* latent, avits_dtype dt, int B, int M,
+                                      int grid_h, int grid_w, int C, int p,
+                                      const int32_t* pos_in_opt, const int32_t* span_in_opt,
+                                      const uint8_t* sel_mask, const int32_t* tok_offset, int k,
+                                      avits_upmode mode, void* out_latent, int32_t* out_pos,
+                                      int32_t* out_span, int32_t* out_src_tok,
+                                      int8_t* out_src_sub, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Final merge, Sec. 3.2 Stage 3: expand every remaining token to full
+ * resolution and lay the tokens out in spatial (raster) order.
+ * A token at (y,x) with span s covers cells [y,y+s) x [x,x+s) of the
+ * full_h x full_w frame; the tokens must tile the frame exactly once
+ * (otherwise AVITS_ERR_COVERAGE is raised on the device).
+ *   nearest  : full-res pixel (Y,X) takes token pixel ((Y-2y)/s, (X-2x)/s).
+ *   bilinear : only for spans {1,2} (one transition): span-1 tokens are
+ *              copied; the low-res grid is rebuilt (span-2 tokens as they are,
+ *              each group of 4 span-1 children 2x2 average pooled) and the
+ *              span-2 cells take its half-pixel-centred 2x bilinear resize.
+ * mixed : [B,N,C*4].  pos [B,N,2], span [B,N] int32.
+ * out_full : [B,full_h*full_w,C*4] same dtype.
+ * workspace : avits_merge_final_workspace() bytes (0 for nearest).
+ * ---------------------------------------------------------------------- */
+avits_status avits_merge_final(const void* mixed, avits_dtype dt, int B, int N,
+                               const int32_t* pos, const int32_t* span, int full_h, int full_w,
+                               int C, int p, avits_upmode mode, void* out_full,
+                               void* workspace, size_t ws_bytes, void* stream);
+
+size_t avits_merge_final_workspace(avits_upmode mode, int B, int full_h, int full_w);
+
+/* ------------------------------------------------------------------------
+ * Synchronises `stream`, returns the OR of the device-side error codes
+ * raised since the last call (as the lowest-numbered set code, or AVITS_OK)
+ * and clears the word.  The only call that blocks the host.
+ * ---------------------------------------------------------------------- */
+avits_status avits_device_status(void* stream);
+
+/* Static text of a status code. */
+const char* avits_status_string(avits_status s);
+
+/* Text of the last CUDA error seen by this thread's calls ("" if none). */
+const char* avits_last_error_string(void);
+
+/* Library version, "MAJOR.MINOR.PATCH". */
+const char* avits_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AVITS_H */
