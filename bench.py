@@ -1,0 +1,574 @@
+#!/usr/bin/env python3
+"""Throughput of the AViTS resolution transition on GB300.
+
+One step = one pass of the whole hot path over one FLUX-1024-shaped transition
+(batch 1): spatial score (Eq. 3-5) -> temporal score -> fuse + top-k
+(Eq. 8-9) -> selective upsample (Stage 2) -> final merge (Stage 3), all on the
+device through the C ABI.  Inputs are resident in HBM; the step rotates over
+NSETS copies of the inputs (> L2) so that no step reads inputs left in L2 by
+the previous ones.  The timed region replays CUDA graphs of those steps.
+
+Prints one JSON line.  --impl reference times the CPU oracle instead.
+Multi-GPU (torchrun): every rank runs an independent replica ("replicas
+only": the path has no exchange step); value = all ranks' transitions / max
+rank time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "transitions/s at FLUX-1024 shape"
+UNIT = "transitions/s"
+WORKLOAD = "flux1024"
+L2_BYTES = 129 * 1024 * 1024
+
+
+def _args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--mode", default="nearest", choices=["nearest", "bilinear"])
+    ap.add_argument("--sets", type=int, default=10, help="input copies rotated per step")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--quick", action="store_true", help="skip the secondary measurements")
+    return ap.parse_args()
+
+
+# ----------------------------------------------------------------- dist ----
+def dist_setup(n_gpus):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        backend = os.environ.get("AVITS_BENCH_BACKEND", "nccl")
+        dist.init_process_group(backend=backend)
+        pg = dist
+    return world, rank, local, pg
+
+
+def barrier(pg):
+    if pg is not None:
+        pg.barrier()
+
+
+def max_over_ranks(pg, value: float, device=None) -> float:
+    """Largest `value` over all ranks (the slowest rank sets the job time)."""
+    if pg is None:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate(units_per_rank: int, world: int, max_seconds: float):
+    """Whole-job throughput: every rank's units over the slowest rank's time."""
+    return units_per_rank * world / max_seconds
+
+
+# --------------------------------------------------------------- clocks ----
+class ClockSampler:
+    """nvidia-smi samples taken while the GPU runs the measured work."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def mark(self):
+        return time.time()
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self, t0: float, t1: float):
+        rows = [l for (t, l) in self.lines if t0 <= t <= t1] or [l for (_, l) in self.lines]
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for l in rows:
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------- roofline inputs ----
+def algorithmic_work(tr, mode):
+    """Per-launch algorithmic FLOPs / bytes of each kernel (one transition)."""
+    elt = 2 if tr.dtype == "bf16" else 4
+    B, H, M, Nk, d, D, T = tr.B, tr.H, tr.M, tr.Nk, tr.d, tr.D, tr.C * 4
+    NO = M + 3 * tr.k
+    F = 4 * tr.frame_h * tr.frame_w
+    return {
+        "spatial": {"flops": 2.0 * B * H * M * Nk * d, "exps": float(B * H * M * Nk),
+                    "bytes": float(B * H * (M + Nk) * d * elt + 4 * B * M)},
+        "temporal": {"bytes": float(2 * B * M * D * elt + 4 * B * M)},
+        "select": {"bytes": float(8 * B * M + 4 * B * M + 4 * B * tr.k + B * M + 4 * B * M)},
+        "upsample": {"bytes": float(B * M * T * elt + B * M * 5 + B * NO * (T * elt + 17))},
+        "merge": {"bytes": float(B * NO * (T * elt + 12) + B * F * T * elt)},
+    }
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p["bf16_tflops"]),
+                "bf16_tflops_sustained": float(p["bf16_tflops_sustained"]), "source": "measured"}
+    except (OSError, KeyError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+def profiled_traffic(kernel_src: str, summary: str):
+    """DRAM bytes per launch recorded by an ncu capture (profiles/), or None
+    when the kernel source changed since that capture."""
+    path = os.path.join(ROOT, "profiles", summary)
+    try:
+        text = open(path).read()
+        with open(kernel_src, "rb") as f:
+            sha = hashlib.sha1(f.read()).hexdigest()[:12]
+    except OSError:
+        return None
+    m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    s = re.search(r"kernel_source_sha1:\s*([0-9a-f]+)", text)
+    if not m or not s or s.group(1) != sha:
+        return None
+    return float(m.group(1))
+
+
+def _smi_id(torch, dev, local):
+    """nvidia-smi -i argument of this rank's GPU (UUID when torch exposes it)."""
+    try:
+        u = str(torch.cuda.get_device_properties(dev).uuid)
+        if u:
+            return u if u.startswith("GPU-") else "GPU-" + u
+    except (AttributeError, RuntimeError):
+        pass
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+    ids = [x for x in vis.split(",") if x.strip()]
+    return ids[local] if local < len(ids) else str(local)
+
+
+# ------------------------------------------------------------------ ours ----
+def run_ours(args, world, rank, local, pg):
+    import torch
+    import paper_2608_17995_gb300 as av
+    from paper_2608_17995_gb300.pipeline import TransitionBuffers, to_device
+    from paper_2608_17995_gb300.workloads import make_transition
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    av.build()
+    av.lib()
+    tr = make_transition(WORKLOAD, seed=1 + 1000 * rank if rank else None)
+    mode = args.mode
+    buf = TransitionBuffers(tr, device=dev, mode=mode, inputs=True)
+    stream = torch.cuda.Stream(device=dev)
+
+    # NSETS resident copies of the inputs, rotated per step (> L2 in total)
+    base = (buf.q, buf.k, buf.h_t, buf.h_prev, buf.latent)
+    set_bytes = sum(t.numel() * t.element_size() for t in base)
+    nsets = max(args.sets, int(math.ceil(2.0 * L2_BYTES / set_bytes)) + 1)
+    sets = [base] + [tuple(t.clone() for t in base) for _ in range(nsets - 1)]
+    torch.cuda.synchronize()
+
+    kernels_per_step = 5 if buf.mode == av.NEAREST else 6   # bilinear merge: map + gather
+    names = ["spatial", "temporal", "select", "upsample", "merge"]
+
+    def step(s, st, events=None):
+        buf.set_inputs(*sets[s % nsets])
+        calls = (buf.spatial, buf.temporal, buf.select, buf.upsample, buf.merge)
+        for i, c in enumerate(calls):
+            if events is not None:
+                events[i].record(st)
+            c(st)
+        if events is not None:
+            events[5].record(st)
+
+    # eager warm-up (also builds the spatial workspace), then graphs
+    with torch.cuda.stream(stream):
+        for s in range(max(args.warmup, 3)):
+            step(s, stream)
+    stream.synchronize()
+    if av.avits_device_status(stream) != 0:
+        raise RuntimeError("device status error during warm-up")
+
+    # one graph runs every input set once (nsets steps); a second graph per
+    # set serves the remainder of K
+    g_all = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_all, stream=stream):
+        for s in range(nsets):
+            step(s, stream)
+    g_one = []
+    for s in range(nsets):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            step(s, stream)
+        g_one.append(g)
+    K, W = args.steps, args.warmup
+
+    def replay_steps(n):
+        full, rem = divmod(n, nsets)
+        for _ in range(full):
+            g_all.replay()
+        for s in range(rem):
+            g_one[s].replay()
+
+    with torch.cuda.stream(stream):
+        replay_steps(max(W, 3))
+    stream.synchronize()
+
+    clocks = ClockSampler(_smi_id(torch, dev, local))
+    clocks.start()
+    time.sleep(0.4)
+    soak_t0 = clocks.mark()
+    # keep the GPU under the same load while the sampler settles (untimed)
+    with torch.cuda.stream(stream):
+        t_end = time.time() + 0.6
+        while time.time() < t_end:
+            replay_steps(nsets)
+            stream.synchronize()
+
+    # ---------------- timed region: exactly K steps ----------------
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    barrier(pg)
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        ev0.record(stream)
+        replay_steps(K)
+        ev1.record(stream)
+    stream.synchronize()
+    torch.cuda.synchronize()
+    barrier(pg)
+    t_ms = ev0.elapsed_time(ev1)
+    clock_t1 = clocks.mark()
+    time.sleep(0.25)
+    clocks.stop()
+    clk = clocks.summary(soak_t0, clock_t1)
+    status = av.avits_device_status(stream)
+    if status != 0:
+        raise RuntimeError("device status %d after the timed region" % status)
+    max_ms = max_over_ranks(pg, t_ms, dev)
+    value = aggregate(K, world, max_ms / 1e3)
+
+    # ---------------- per-kernel durations (events between kernels) ----------
+    per_kernel = per_kernel_times(torch, av, step, nsets, stream, names, args)
+    work = algorithmic_work(tr, mode)
+    peaks = measured_peaks()
+    kt = {}
+    for n in names:
+        ms = per_kernel.get(n)
+        if ms is None:
+            continue
+        e = {"us": round(ms * 1e3, 3)}
+        w = work[n]
+        if "flops" in w:
+            e["tflops"] = round(w["flops"] / (ms * 1e-3) / 1e12, 2)
+            e["frac_tensor"] = round(e["tflops"] / peaks["bf16_tflops"], 4)
+            e["gexp_per_s"] = round(w["exps"] / (ms * 1e-3) / 1e9, 1)
+        e["gbs"] = round(w["bytes"] / (ms * 1e-3) / 1e9, 1)
+        e["frac_hbm"] = round(e["gbs"] / peaks["hbm_gbs"], 4)
+        kt[n] = e
+    sp_ms = per_kernel.get("spatial")
+    traffic = profiled_traffic(os.path.join(ROOT, "paper_2608_17995_gb300", "csrc", "spatial_tc.cu"),
+                               "spatial_tc_flux1024.md")
+    roofline = None
+    if sp_ms:
+        achieved = work["spatial"]["flops"] / (sp_ms * 1e-3) / 1e12
+        roofline = {"kernel": "spatial_tc_kernel (avits_score_spatial)", "bound": "tensor",
+                    "achieved": round(achieved, 2), "peak": peaks["bf16_tflops"],
+                    "unit": "TFLOP/s", "frac": round(achieved / peaks["bf16_tflops"], 4),
+                    "peak_source": peaks["source"] + " bf16 burst (MEASURED_PEAKS.json)",
+                    "traffic": traffic}
+
+    result = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+        "steps": K, "warmup": W, "ms_per_step": round(max_ms / K, 6),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": "FLUX-1024-shaped transition: 32x32 -> 64x64 tokens, 512 text "
+                               "keys, H=24, d=128, D=3072, C=16 p=2, bf16, alpha=0.5, k=307, "
+                               "batch 1, seed 1 (" + mode + " upsample)",
+                   "global_batch": world, "parallelism": "replicas x%d" % world,
+                   "l2": "inputs rotated over %d resident copies (%.0f MB > 129 MB L2)"
+                         % (nsets, nsets * set_bytes / 1e6),
+                   "timing": "CUDA-graph replay of K steps, CUDA events on the launching stream"},
+        "gpu_launches": K * kernels_per_step,
+        "clocks": clk,
+        "kernels": kt,
+        "roofline": roofline,
+    }
+    if not args.no_e2e and not args.quick:
+        result["e2e"] = e2e_measure(torch, av, buf, tr, stream, K, W, world, pg, dev)
+    if mode == "nearest" and not args.quick:
+        result["bilinear"] = mode_measure(torch, av, tr, dev, stream, sets, nsets, K)
+    return result, tr
+
+
+def per_kernel_times(torch, av, step, nsets, stream, names, args):
+    """Average device time of each kernel: a graph of steps with external
+    event-record nodes between the launches (eager with a leading sleep if
+    this torch cannot capture external events)."""
+    n_steps = max(nsets * 10, 100)
+    try:
+        evs = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(6)]
+               for _ in range(n_steps)]
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for s in range(n_steps):
+                step(s, stream, evs[s])
+        with torch.cuda.stream(stream):
+            g.replay()
+            stream.synchronize()
+            g.replay()
+        stream.synchronize()
+        how = "graph"
+    except (TypeError, RuntimeError):
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(n_steps)]
+        with torch.cuda.stream(stream):
+            for s in range(n_steps):
+                torch.cuda._sleep(2_000_000)   # host enqueues the step while the GPU waits
+                step(s, stream, evs[s])
+        stream.synchronize()
+        how = "eager"
+    out = {"_how": how}
+    for i, n in enumerate(names):
+        out[n] = sum(evs[s][i].elapsed_time(evs[s][i + 1]) for s in range(n_steps)) / n_steps
+    return out
+
+
+def mode_measure(torch, av, tr, dev, stream, sets, nsets, K):
+    """Step time with bilinear upsampling / merge (same inputs, graph replay)."""
+    from paper_2608_17995_gb300.pipeline import TransitionBuffers
+    b2 = TransitionBuffers(tr, device=dev, mode="bilinear", inputs=False)
+
+    def step(s):
+        b2.set_inputs(*sets[s % nsets])
+        b2.run(stream)
+
+    with torch.cuda.stream(stream):
+        for s in range(3):
+            step(s)
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for s in range(nsets):
+            step(s)
+    reps = max(1, K // nsets)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        g.replay()
+        e0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        e1.record(stream)
+    stream.synchronize()
+    ms = e0.elapsed_time(e1) / (reps * nsets)
+    st = av.avits_device_status(stream)
+    return {"ms_per_step": round(ms, 6), "value": round(1e3 / ms, 1), "unit": UNIT,
+            "status": st}
+
+
+def e2e_measure(torch, av, buf, tr, stream, K, W, world, pg, dev):
+    """Same metric through the public API from pinned HOST buffers: each step
+    copies its inputs host->device, runs the five calls and reads the merged
+    latent and the selected indices back; graph-captured, CUDA events."""
+    inputs = (buf.q, buf.k, buf.h_t, buf.h_prev, buf.latent)
+    host_in = [t.cpu().pin_memory() for t in inputs]
+    dev_in = [torch.empty_like(t) for t in inputs]
+    host_full = torch.empty(buf.full.shape, dtype=buf.full.dtype).pin_memory()
+    host_sel = torch.empty(buf.sel_idx.shape, dtype=buf.sel_idx.dtype).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in host_in)
+    d2h = host_full.numel() * host_full.element_size() + host_sel.numel() * host_sel.element_size()
+
+    def step():
+        for d, h in zip(dev_in, host_in):
+            d.copy_(h, non_blocking=True)
+        buf.set_inputs(*dev_in)
+        buf.run(stream)
+        host_full.copy_(buf.full, non_blocking=True)
+        host_sel.copy_(buf.sel_idx, non_blocking=True)
+
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            step()
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        step()
+    n = max(10, min(K, 500))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            g.replay()
+        barrier(pg)
+        e0.record(stream)
+        for _ in range(n):
+            g.replay()
+        e1.record(stream)
+    stream.synchronize()
+    barrier(pg)
+    ms = max_over_ranks(pg, e0.elapsed_time(e1), dev)
+    return {"value": round(aggregate(n, world, ms / 1e3), 1), "unit": UNIT,
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": n,
+            "ms_per_step": round(ms / n, 6)}
+
+
+# ---------------------------------------------------------- CPU oracle ----
+def oracle_transition_sample(tr, rows, orc):
+    """The oracle's transition with the spatial score on a row sample."""
+    t0 = time.perf_counter()
+    A, _, _ = orc.score_spatial(tr.q_img, tr.k_all, tr.L, tr.softmax_scale, rows=rows)
+    t1 = time.perf_counter()
+    V = orc.score_temporal(tr.h_t, tr.h_prev)
+    S = orc.fuse(A, V, tr.alpha)
+    sel, mask, off = orc.topk(S, tr.k)
+    out, pos, span, _, _ = orc.selective_upsample(tr.latent, tr.grid_h, tr.grid_w, mask)
+    orc.merge_final(out, pos, span, 2 * tr.grid_h, 2 * tr.grid_w)
+    t2 = time.perf_counter()
+    return t1 - t0, t2 - t1
+
+
+def cpu_baseline(tr, budget_s=15.0, frac=16):
+    """Oracle throughput on this host's cores: each sample scores 1/frac of
+    the image rows (all heads, all keys) and runs the rest of the path in
+    full; a transition is costed as frac x the sampled spatial time plus the
+    rest.  Repeats until ~budget_s of CPU work."""
+    import numpy as np
+    import oracle as orc
+    orc.build()
+    rows = np.arange(0, tr.B * tr.M, frac, dtype=np.int32)
+    tsp, trest, n = 0.0, 0.0, 0
+    t_start = time.perf_counter()
+    while True:
+        a, b = oracle_transition_sample(tr, rows, orc)
+        tsp += a
+        trest += b
+        n += 1
+        if time.perf_counter() - t_start > budget_s or n >= 50:
+            break
+    per_transition = frac * tsp / n + trest / n
+    return {"value": round(1.0 / per_transition, 4), "unit": UNIT, "cores": orc.threads(),
+            "kind": "oracle",
+            "sample": "%d samples of the FLUX-1024 transition, each with the spatial score on "
+                      "1/%d of the image rows (%d rows x 24 heads x 1536 keys) and the temporal "
+                      "score, fuse+top-k, upsample and merge in full; transition time = %d x "
+                      "spatial sample + rest" % (n, frac, len(rows), frac)}
+
+
+def run_reference(args, world, rank, pg):
+    """The oracle timed as it stands (bench's reference arm)."""
+    from paper_2608_17995_gb300.workloads import make_transition
+    import numpy as np
+    import oracle as orc
+    orc.build()
+    if rank != 0:
+        return None
+    tr = make_transition(WORKLOAD)
+    frac = 64
+    rows = np.arange(0, tr.B * tr.M, frac, dtype=np.int32)
+    for _ in range(args.warmup):
+        oracle_transition_sample(tr, rows, orc)
+    tsp, trest = 0.0, 0.0
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        a, b = oracle_transition_sample(tr, rows, orc)
+        tsp += a
+        trest += b
+    wall = time.perf_counter() - t0
+    per = frac * tsp / args.steps + trest / args.steps
+    value = 1.0 / per
+    sample = ("each step: the oracle transition with the spatial score on 1/%d of the image rows "
+              "(%d rows, all heads and keys) and the rest of the path in full; transition time = "
+              "%d x spatial sample + rest" % (frac, len(rows), frac))
+    return {"impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(per * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": "FLUX-1024-shaped transition (oracle, CPU)",
+                       "wall_s": round(wall, 2)},
+            "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": orc.threads(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def main():
+    args = _args()
+    world, rank, local, pg = dist_setup(args.gpus)
+    if args.impl == "reference":
+        res = run_reference(args, world, rank, pg)
+        if res is not None:
+            print(json.dumps(res), flush=True)
+        if pg is not None:
+            pg.destroy_process_group()
+        return 0
+    res, tr = run_ours(args, world, rank, local, pg)
+    if rank == 0:
+        if world == 1 and not args.no_cpu_baseline:
+            res["cpu_baseline"] = cpu_baseline(tr)
+        print(json.dumps(res), flush=True)
+    if pg is not None:
+        pg.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,259 @@
+"""AViTS resolution-transition hot path for GB300 (sm_103a).
+
+A thin ctypes binding over ``libavits.so`` (include/avits.h).  Each function
+has the name of its C entry point and only marshals arguments: torch tensors
+become device pointers, the current torch stream becomes the cudaStream_t, a
+non-OK status becomes an ``AvitsError``.  Every step of the path runs in the
+library's CUDA kernels; there is no CPU fallback, and importing the functions
+fails loudly when the library has not been built (``build()``).
+
+Calls:
+  avits_score_spatial       Eq. 3-5  text attention mass per image token
+  avits_score_temporal      Sec. 3.3.2  relative step change per token
+  avits_score_temporal_var  Eq. 6-7  step variance over N_T snapshots
+  avits_fuse_select         Eq. 8-9  min-max fuse + deterministic top-k
+  avits_selective_upsample  Sec. 3.2 Stage 2  packed mixed-resolution sequence
+  avits_merge_final         Sec. 3.2 Stage 3  dense full-resolution latent
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence
+
+from . import _build
+
+__all__ = [
+    "AvitsError", "build", "lib", "library_path",
+    "avits_score_spatial", "avits_score_spatial_workspace", "avits_score_temporal",
+    "avits_score_temporal_var", "avits_fuse_select", "avits_selective_upsample",
+    "avits_merge_final", "avits_merge_final_workspace", "avits_device_status",
+    "avits_status_string", "avits_version", "SpatialWorkspace",
+]
+
+F32, BF16 = 0, 1
+NEAREST, BILINEAR = 0, 1
+STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported", 3: "CUDA error",
+          4: "device wait timed out", 5: "NaN in fused score", 6: "coverage"}
+
+_lib = None
+
+
+class AvitsError(RuntimeError):
+    def __init__(self, fn: str, code: int, detail: str = ""):
+        self.code = code
+        super().__init__("%s failed: %s%s" % (fn, STATUS.get(code, code),
+                                               (" (" + detail + ")") if detail else ""))
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def build(force: bool = False) -> str:
+    """Compile libavits.so for sm_103a (in-tree)."""
+    return _build.build(force=force)
+
+
+def lib():
+    """Load libavits.so; raise if it is missing (no fallback path exists)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.LIB
+    if not os.path.exists(path):
+        raise RuntimeError("libavits.so is not built (%s); run paper_2608_17995_gb300.build()" % path)
+    L = ctypes.CDLL(path)
+    vp, i32, i64, f32, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
+    sig = {
+        "avits_score_spatial": [vp, vp, i32, i32, i32, i32, i32, i32, i32, i64, i64, i64, i64, i64,
+                                i64, f32, f32, i32, vp, vp, vp, sz, vp],
+        "avits_score_spatial_workspace": [i32, i32, i32, i32, i32, i32],
+        "avits_score_temporal": [vp, vp, i32, i32, i32, i32, f32, vp, vp],
+        "avits_score_temporal_var": [vp, i32, i32, i32, i32, i32, vp, vp],
+        "avits_fuse_select": [vp, vp, i32, i32, f32, f32, i32, vp, vp, vp, vp, vp],
+        "avits_selective_upsample": [vp, i32, i32, i32, i32, i32, i32, i32, vp, vp, vp, vp, i32,
+                                     i32, vp, vp, vp, vp, vp, vp],
+        "avits_merge_final": [vp, i32, i32, i32, vp, vp, i32, i32, i32, i32, i32, vp, vp, sz, vp],
+        "avits_merge_final_workspace": [i32, i32, i32, i32],
+        "avits_device_status": [vp],
+        "avits_status_string": [i32],
+        "avits_last_error_string": [],
+        "avits_version": [],
+    }
+    for name, args in sig.items():
+        fn = getattr(L, name)
+        fn.argtypes = args
+        fn.restype = ctypes.c_int
+    for name in ("avits_score_spatial_workspace", "avits_merge_final_workspace"):
+        getattr(L, name).restype = ctypes.c_size_t
+    for name in ("avits_status_string", "avits_last_error_string", "avits_version"):
+        getattr(L, name).restype = ctypes.c_char_p
+    _lib = L
+    return L
+
+
+# ------------------------------------------------------------- marshalling --
+def _torch():
+    import torch
+    return torch
+
+
+def _ptr(t) -> Optional[int]:
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    if not t.is_cuda:
+        raise ValueError("device tensor expected, got a %s tensor" % t.device)
+    return t.data_ptr()
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        return _torch().cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _dtype_code(t) -> int:
+    torch = _torch()
+    if t.dtype == torch.bfloat16:
+        return BF16
+    if t.dtype == torch.float32:
+        return F32
+    raise TypeError("bfloat16 or float32 expected, got %s" % t.dtype)
+
+
+def _check(fn: str, rc: int):
+    if rc != 0:
+        detail = lib().avits_last_error_string().decode() if rc == 3 else ""
+        raise AvitsError(fn, rc, detail)
+
+
+def avits_version() -> str:
+    return lib().avits_version().decode()
+
+
+def avits_status_string(code: int) -> str:
+    return lib().avits_status_string(code).decode()
+
+
+def avits_device_status(stream=None) -> int:
+    """Synchronise the stream; return and clear the device error code (0 = ok)."""
+    return lib().avits_device_status(_stream(stream))
+
+
+def avits_score_spatial_workspace(dtype, B, H, M, Nk, d) -> int:
+    code = dtype if isinstance(dtype, int) else _dtype_code(_torch().empty(0, dtype=dtype))
+    return int(lib().avits_score_spatial_workspace(code, B, H, M, Nk, d))
+
+
+class SpatialWorkspace:
+    """A zero-filled device buffer for avits_score_spatial, grown on demand.
+    The kernels leave it zero-filled after every successful call."""
+
+    def __init__(self, device=None):
+        self.buf = None
+        self.device = device
+
+    def get(self, nbytes: int):
+        torch = _torch()
+        if nbytes == 0:
+            return None, 0
+        if self.buf is None or self.buf.numel() < nbytes:
+            self.buf = torch.zeros(nbytes, dtype=torch.uint8, device=self.device or "cuda")
+        return self.buf, self.buf.numel()
+
+    def reset(self):
+        if self.buf is not None:
+            self.buf.zero_()
+
+
+_default_ws = {}
+
+
+def avits_score_spatial(q_img, k_all, L: int, softmax_scale: float, A, weight: float = 1.0,
+                        accumulate: bool = False, lse=None, workspace: Optional[SpatialWorkspace] = None,
+                        stream=None):
+    """Eq. 3-5.  q_img [B,H,M,d] (any strides, d contiguous), k_all [B,H,Nk,d]
+    with the L text keys first; A [B,M] fp32 written (or accumulated)."""
+    B, H, M, d = q_img.shape
+    Nk = k_all.shape[2]
+    if k_all.shape[0] != B or k_all.shape[1] != H or k_all.shape[3] != d:
+        raise ValueError("q_img / k_all shapes disagree")
+    if q_img.stride(3) != 1 or k_all.stride(3) != 1:
+        raise ValueError("the head-dim axis must be contiguous")
+    dt = _dtype_code(q_img)
+    if _dtype_code(k_all) != dt:
+        raise TypeError("q_img and k_all dtypes differ")
+    need = int(lib().avits_score_spatial_workspace(dt, B, H, M, Nk, d))
+    if workspace is None:
+        key = (q_img.device.index, _torch().cuda.current_stream().cuda_stream if stream is None else _stream(stream))
+        workspace = _default_ws.setdefault(key, SpatialWorkspace(q_img.device))
+    wbuf, wbytes = workspace.get(need)
+    rc = lib().avits_score_spatial(
+        _ptr(q_img), _ptr(k_all), dt, B, H, M, Nk, L, d,
+        q_img.stride(0), q_img.stride(1), q_img.stride(2),
+        k_all.stride(0), k_all.stride(1), k_all.stride(2),
+        float(softmax_scale), float(weight), 1 if accumulate else 0,
+        _ptr(A), _ptr(lse), _ptr(wbuf), wbytes, _stream(stream))
+    _check("avits_score_spatial", rc)
+    return A
+
+
+def avits_score_temporal(h_t, h_prev, V, eps: float = 1e-6, stream=None):
+    B, N, D = h_t.shape
+    if not (h_t.is_contiguous() and h_prev.is_contiguous()):
+        raise ValueError("h_t and h_prev must be contiguous")
+    rc = lib().avits_score_temporal(_ptr(h_t), _ptr(h_prev), _dtype_code(h_t), B, N, D,
+                                    float(eps), _ptr(V), _stream(stream))
+    _check("avits_score_temporal", rc)
+    return V
+
+
+def avits_score_temporal_var(snaps: Sequence, V, stream=None):
+    B, N, D = snaps[0].shape
+    arr = (ctypes.c_void_p * len(snaps))(*[_ptr(s) for s in snaps])
+    rc = lib().avits_score_temporal_var(arr, len(snaps), _dtype_code(snaps[0]), B, N, D, _ptr(V),
+                                        _stream(stream))
+    _check("avits_score_temporal_var", rc)
+    return V
+
+
+def avits_fuse_select(A, V, alpha: float, k: int, sel_idx, tok_offset, S=None, sel_mask=None,
+                      eps_norm: float = 1e-6, stream=None):
+    B, M = A.shape
+    rc = lib().avits_fuse_select(_ptr(A), _ptr(V), B, M, float(alpha), float(eps_norm), int(k),
+                                 _ptr(S), _ptr(sel_idx), _ptr(sel_mask), _ptr(tok_offset),
+                                 _stream(stream))
+    _check("avits_fuse_select", rc)
+    return sel_idx
+
+
+def avits_selective_upsample(latent, grid_h: int, grid_w: int, sel_mask, tok_offset, k: int,
+                             out_latent, out_pos, out_span, out_src_tok, out_src_sub,
+                             mode: int = NEAREST, pos_in=None, span_in=None, stream=None):
+    B, M, T = latent.shape
+    rc = lib().avits_selective_upsample(
+        _ptr(latent), _dtype_code(latent), B, M, grid_h, grid_w, T // 4, 2, _ptr(pos_in),
+        _ptr(span_in), _ptr(sel_mask), _ptr(tok_offset), int(k), int(mode), _ptr(out_latent),
+        _ptr(out_pos), _ptr(out_span), _ptr(out_src_tok), _ptr(out_src_sub), _stream(stream))
+    _check("avits_selective_upsample", rc)
+    return out_latent
+
+
+def avits_merge_final_workspace(mode: int, B: int, full_h: int, full_w: int) -> int:
+    return int(lib().avits_merge_final_workspace(int(mode), B, full_h, full_w))
+
+
+def avits_merge_final(mixed, pos, span, full_h: int, full_w: int, out_full, mode: int = NEAREST,
+                      workspace=None, stream=None):
+    B, N, T = mixed.shape
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    rc = lib().avits_merge_final(_ptr(mixed), _dtype_code(mixed), B, N, _ptr(pos), _ptr(span),
+                                 full_h, full_w, T // 4, 2, int(mode), _ptr(out_full),
+                                 _ptr(workspace), ws_bytes, _stream(stream))
+    _check("avits_merge_final", rc)
+    return out_full

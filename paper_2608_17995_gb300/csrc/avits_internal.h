@@ -1,0 +1,65 @@
+// avits_internal.h — launchers behind the C ABI (host side, not exported).
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "avits.h"
+
+namespace avits {
+
+// Device address of the status word of the current device (api.cu).
+unsigned int* status_word();
+
+// ---- spatial (Eq. 3-5) ------------------------------------------------------
+struct SpatialArgs {
+  const void* q;
+  const void* k;
+  avits_dtype dt;
+  int B, H, M, Nk, L, d;
+  int64_t q_sb, q_sh, q_sn, k_sb, k_sh, k_sn;   // element strides
+  float scale, weight;
+  int accumulate;
+  float* A;
+  float* lse;
+  void* ws;
+  size_t ws_bytes;
+  unsigned int* status;
+};
+
+// tcgen05 / TMA path (bf16, d in {64,128}); returns false if the shape or
+// layout is not eligible (the caller then uses the CUDA-core path).
+bool spatial_tc_eligible(const SpatialArgs& a);
+size_t spatial_tc_workspace(int B, int H, int M, int Nk, int d, int num_sms);
+cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s);
+
+// CUDA-core path (fp32 or bf16, any d <= 256): one warp per query row.
+cudaError_t launch_spatial_simt(const SpatialArgs& a, cudaStream_t s);
+
+// ---- temporal ---------------------------------------------------------------
+cudaError_t launch_temporal(const void* ht, const void* hp, avits_dtype dt, int B, int N, int D,
+                            float eps, float* V, int num_sms, cudaStream_t s);
+constexpr int kMaxSnapshots = 16;
+cudaError_t launch_temporal_var(const void* const* snaps, int n_t, avits_dtype dt, int B, int N,
+                                int D, float* V, int num_sms, cudaStream_t s);
+
+// ---- fuse + select (Eq. 8-9) ------------------------------------------------
+constexpr int kSelectMaxM = 32768;
+cudaError_t launch_fuse_select(const float* A, const float* V, int B, int M, float alpha,
+                               float eps, int k, float* S, int32_t* sel_idx, uint8_t* mask,
+                               int32_t* tok_offset, unsigned int* status, cudaStream_t s);
+
+// ---- selective upsample (Stage 2) -------------------------------------------
+cudaError_t launch_upsample(const void* latent, avits_dtype dt, int B, int M, int gh, int gw,
+                            int C, const int32_t* pos_in, const int32_t* span_in,
+                            const uint8_t* mask, const int32_t* tok_offset, int k,
+                            avits_upmode mode, void* out, int32_t* out_pos, int32_t* out_span,
+                            int32_t* out_src_tok, int8_t* out_src_sub, cudaStream_t s);
+
+// ---- final merge (Stage 3) --------------------------------------------------
+cudaError_t launch_merge(const void* mixed, avits_dtype dt, int B, int N, const int32_t* pos,
+                         const int32_t* span, int fh, int fw, int C, avits_upmode mode,
+                         void* out, void* ws, unsigned int* status, cudaStream_t s);
+
+}  // namespace avits

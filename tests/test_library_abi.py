@@ -1,0 +1,97 @@
+"""Host-side checks of the C ABI (no GPU needed): the library builds for
+sm_103a, exports every symbol include/avits.h declares, and rejects bad
+arguments on the host without launching anything."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    import paper_2608_17995_gb300 as av
+    av.build()
+    return av.lib()
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "avits.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(avits_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = declared_functions()
+    assert len(names) >= 12
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_static_strings(lib):
+    assert lib.avits_version().decode().count(".") == 2
+    assert lib.avits_status_string(0) == b"ok"
+    assert b"timed out" in lib.avits_status_string(4)
+
+
+def test_host_validation_rejects_without_launch(lib):
+    P = ctypes.c_void_p(16)          # a non-null, 16-byte aligned dummy pointer
+    INVALID, UNSUPPORTED = 1, 2
+    # k > M
+    assert lib.avits_fuse_select(P, P, 1, 10, 0.5, 1e-6, 11, None, P, None, P, None) == INVALID
+    # alpha outside [0,1]
+    assert lib.avits_fuse_select(P, P, 1, 10, 1.5, 1e-6, 3, None, P, None, P, None) == INVALID
+    # M above the single-CTA selection limit
+    assert lib.avits_fuse_select(P, P, 1, 40000, 0.5, 1e-6, 3, None, P, None, P, None) == INVALID
+    # L > Nk, non-positive scale, row stride shorter than d
+    args = [P, P, 1, 1, 2, 64, 96, 97, 64, 0, 0, 64, 0, 0, 64, 0.125, 1.0, 0, P, None, None, 0, None]
+    assert lib.avits_score_spatial(*args) == INVALID
+    args[7] = 32
+    args[15] = 0.0
+    assert lib.avits_score_spatial(*args) == INVALID
+    args[15] = 0.125
+    args[11] = 32
+    assert lib.avits_score_spatial(*args) == INVALID
+    # temporal: empty token range, too many snapshots
+    assert lib.avits_score_temporal(P, P, 1, 1, 0, 64, 1e-6, P, None) == INVALID
+    snaps = (ctypes.c_void_p * 17)(*([16] * 17))
+    assert lib.avits_score_temporal_var(snaps, 17, 1, 1, 4, 8, P, None) == INVALID
+    # upsample: patch size other than 2, grid that does not match M, bilinear on mixed input
+    up = [P, 1, 1, 16, 4, 4, 16, 2, None, None, P, P, 4, 0, P, P, P, P, P, None]
+    up[7] = 3
+    assert lib.avits_selective_upsample(*up) == UNSUPPORTED
+    up[7] = 2
+    up[4] = 5
+    assert lib.avits_selective_upsample(*up) == INVALID
+    up[4] = 4
+    up[8], up[9], up[13] = P, P, 1
+    assert lib.avits_selective_upsample(*up) == UNSUPPORTED
+    # merge: bilinear needs an even frame and a workspace; misaligned output
+    mg = [P, 1, 1, 28, P, P, 8, 8, 1, 2, 1, P, None, 0, None]
+    assert lib.avits_merge_final(*mg) == INVALID
+    mg[12], mg[13] = P, 1 << 20
+    mg[6] = 7
+    assert lib.avits_merge_final(*mg) == INVALID
+    mg[6] = 8
+    mg[11] = ctypes.c_void_p(24)
+    assert lib.avits_merge_final(*mg) == INVALID
+
+
+def test_workspace_queries(lib):
+    assert lib.avits_merge_final_workspace(0, 1, 64, 64) == 0
+    assert lib.avits_merge_final_workspace(1, 2, 64, 64) == 2 * 64 * 64 * 4
+    assert lib.avits_score_spatial_workspace(0, 1, 2, 256, 288, 64) == 0   # fp32: no workspace
+    assert lib.avits_score_spatial_workspace(1, 1, 24, 1024, 1536, 128) > 0
+
+
+def test_product_path_does_not_touch_the_oracle():
+    """The package never imports the oracle (only tests, smoke and the bench
+    baseline may)."""
+    pkg = os.path.join(ROOT, "paper_2608_17995_gb300")
+    for dp, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                text = open(os.path.join(dp, f)).read()
+                assert "import oracle" not in text and "avits_oracle" not in text, f
