@@ -353,6 +353,8 @@ def run_ours(args, world, rank, local, pg):
         "gpu_launches": K * kernels_per_step,
         "clocks": clk,
         "kernels": kt,
+        "kernels_timing": {"how": per_kernel["_how"],
+                           "eager_step_us": round(per_kernel["_step"] * 1e3, 3)},
         "roofline": roofline,
     }
     if not args.no_e2e and not args.quick:
@@ -363,34 +365,20 @@ def run_ours(args, world, rank, local, pg):
 
 
 def per_kernel_times(torch, av, step, nsets, stream, names, args):
-    """Average device time of each kernel: a graph of steps with external
-    event-record nodes between the launches (eager with a leading sleep if
-    this torch cannot capture external events)."""
+    """Average device time of each kernel over eager steps whose launches
+    are all queued behind a sleep kernel, so that the events between them
+    bracket back-to-back kernels rather than host launch latency."""
     n_steps = max(nsets * 10, 100)
-    try:
-        evs = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(6)]
-               for _ in range(n_steps)]
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=stream):
-            for s in range(n_steps):
-                step(s, stream, evs[s])
-        with torch.cuda.stream(stream):
-            g.replay()
-            stream.synchronize()
-            g.replay()
-        stream.synchronize()
-        how = "graph"
-    except (TypeError, RuntimeError):
-        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(n_steps)]
-        with torch.cuda.stream(stream):
-            for s in range(n_steps):
-                torch.cuda._sleep(2_000_000)   # host enqueues the step while the GPU waits
-                step(s, stream, evs[s])
-        stream.synchronize()
-        how = "eager"
-    out = {"_how": how}
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(n_steps)]
+    with torch.cuda.stream(stream):
+        for s in range(n_steps):
+            torch.cuda._sleep(1_000_000)     # ~0.5 ms: the host enqueues the step meanwhile
+            step(s, stream, evs[s])
+    stream.synchronize()
+    out = {"_how": "eager, queued behind a sleep kernel"}
     for i, n in enumerate(names):
         out[n] = sum(evs[s][i].elapsed_time(evs[s][i + 1]) for s in range(n_steps)) / n_steps
+    out["_step"] = sum(evs[s][0].elapsed_time(evs[s][5]) for s in range(n_steps)) / n_steps
     return out
 
 
