@@ -91,10 +91,12 @@ typedef enum { AVITS_UP_NEAREST = 0, AVITS_UP_BILINEAR = 1 } avits_upmode;
  * lse_opt : NULL or [B,H,M,2] fp32 receiving (log sum_j exp l_ij over all
  *         keys, the same over the text keys), natural log; -inf when a sum
  *         underflows.
- * workspace/ws_bytes : at least avits_score_spatial_workspace(...) bytes.
- *         It MUST be zero-filled before its first use; every successful
- *         call leaves it zero-filled again.  After a device error re-zero it.
- *         One workspace must not be used by two calls running concurrently.
+ * workspace/ws_bytes : at least avits_score_spatial_workspace(...) bytes of
+ *         device scratch (per-row partial statistics of the key ranges each
+ *         SM handled; no initial contents are needed).  One workspace must
+ *         not be used by two calls running concurrently.  The bf16
+ *         tensor-core path runs two kernels (scores, then a merge launched
+ *         as a programmatic dependent on the same stream).
  * ---------------------------------------------------------------------- */
 avits_status avits_score_spatial(const void* q_img, const void* k_all, avits_dtype dt,
                                  int B, int H, int M, int Nk, int L, int d,

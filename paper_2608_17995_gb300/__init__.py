@@ -151,8 +151,8 @@ def avits_score_spatial_workspace(dtype, B, H, M, Nk, d) -> int:
 
 
 class SpatialWorkspace:
-    """A zero-filled device buffer for avits_score_spatial, grown on demand.
-    The kernels leave it zero-filled after every successful call."""
+    """Device scratch for avits_score_spatial, grown on demand (reused by
+    calls on one stream; its contents need no initialisation)."""
 
     def __init__(self, device=None):
         self.buf = None
@@ -163,7 +163,7 @@ class SpatialWorkspace:
         if nbytes == 0:
             return None, 0
         if self.buf is None or self.buf.numel() < nbytes:
-            self.buf = torch.zeros(nbytes, dtype=torch.uint8, device=self.device or "cuda")
+            self.buf = torch.empty(nbytes, dtype=torch.uint8, device=self.device or "cuda")
         return self.buf, self.buf.numel()
 
     def reset(self):

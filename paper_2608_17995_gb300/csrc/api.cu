@@ -115,7 +115,7 @@ avits_status avits_score_temporal(const void* h_t, const void* h_prev, avits_dty
   if (!h_t || !h_prev || !V || !valid_dtype(dt)) return AVITS_ERR_INVALID_ARG;
   if (B <= 0 || N <= 0 || D <= 0 || !(eps >= 0.f)) return AVITS_ERR_INVALID_ARG;
   return cuda_status(launch_temporal(h_t, h_prev, dt, B, N, D, eps, V, num_sms_current(),
-                                     static_cast<cudaStream_t>(stream)));
+                                     status_word(), static_cast<cudaStream_t>(stream)));
 }
 
 avits_status avits_score_temporal_var(const void* const* snaps, int n_t, avits_dtype dt, int B,

@@ -39,7 +39,7 @@ cudaError_t launch_spatial_simt(const SpatialArgs& a, cudaStream_t s);
 
 // ---- temporal ---------------------------------------------------------------
 cudaError_t launch_temporal(const void* ht, const void* hp, avits_dtype dt, int B, int N, int D,
-                            float eps, float* V, int num_sms, cudaStream_t s);
+                            float eps, float* V, int num_sms, unsigned int* status, cudaStream_t s);
 constexpr int kMaxSnapshots = 16;
 cudaError_t launch_temporal_var(const void* const* snaps, int n_t, avits_dtype dt, int B, int N,
                                 int D, float* V, int num_sms, cudaStream_t s);

@@ -1,26 +1,35 @@
 // select.cu — joint score and token selection (Sec. 3.3.3, Eq. 8-9).
 //
-// One CTA of 1024 threads per batch element; the M scores stay in shared
-// memory as order-preserving 32-bit keys.
-//   1. min / max of A and V (NaN ignored), block reduction;
+// One CTA of 512 threads per batch element, few barriers:
+//   1. min / max of A and V (NaN ignored): warp shuffles, one shared-memory
+//      round, every warp finishes the reduction itself;
 //   2. S = (alpha * A^) + ((1 - alpha) * V^) with explicitly rounded fp32
 //      operations in that order (no contraction), so that the same A, V give
-//      bit-identical S wherever the selection is recomputed;
-//   3. the k-th largest key by MSB-first radix select, 4 passes of 8 bits
-//      with a 256-bin shared histogram;
-//   4. keys above it are selected, and among keys equal to it the lowest
-//      indices (a block scan over contiguous per-thread ranges);
-//   5. a second block scan yields sel_idx (ascending) and tok_offset.
-// Key map: NaN -> 0 (below everything); -0 -> +0; otherwise the IEEE bits
-// with the sign bit flipped (positive) or all bits flipped (negative).
+//      bit-identical S wherever the selection is recomputed; each S becomes
+//      an order-preserving 32-bit key (NaN -> 0, below everything; -0 -> +0;
+//      otherwise the IEEE bits with the sign bit flipped if positive, all
+//      bits flipped if negative), kept in registers and in shared memory;
+//   3. the k-th largest key by MSB-first radix select with 4-bit digits:
+//      each warp counts its keys per digit with ballots (lane j < 16 counts
+//      digit j; no shared-memory atomics, which would all hit one bin since
+//      scores in [0,1] share their top key bits), the per-warp counts go to a
+//      double-buffered table and every warp scans the 16 digits itself, so a
+//      pass costs one barrier; the passes stop once the k-th key's digit is
+//      taken whole;
+//   4. selection over contiguous per-thread index ranges with ONE block scan
+//      of (keys above the threshold, keys equal to it): the equal keys are
+//      taken lowest index first, so a thread's selected-before count is
+//      above_before + min(r, equal_before) for the r equal keys still needed;
+//      it yields sel_idx (ascending), the mask and tok_offset.
 #include "avits_common.cuh"
 #include "avits_internal.h"
 
 namespace avits {
 namespace {
 
-constexpr int kThreads = 1024;
+constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
+constexpr int kMaxRegKeys = 8;   // keys per thread kept in registers (M <= 4096)
 
 __device__ __forceinline__ uint32_t order_key(float s) {
   if (s != s) return 0u;
@@ -29,36 +38,27 @@ __device__ __forceinline__ uint32_t order_key(float s) {
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-// Exclusive prefix sum over the block (thread order); returns the total.
-__device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* warp_tot,
-                                                         uint32_t* excl) {
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  uint32_t x = v;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
-    if (lane >= o) x += y;
-  }
-  if (lane == 31) warp_tot[w] = x;
-  __syncthreads();
-  if (w == 0) {
-    uint32_t t = warp_tot[lane];
-    uint32_t s = t;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t y = __shfl_up_sync(0xffffffffu, s, o);
-      if (lane >= o) s += y;
-    }
-    warp_tot[lane] = s - t;        // exclusive over warps
-    if (lane == 31) warp_tot[32] = s;
-  }
-  __syncthreads();
-  *excl = warp_tot[w] + x - v;
-  const uint32_t total = warp_tot[32];
-  __syncthreads();
-  return total;
+// Per-warp digit counts of the keys matching `prefix` on `pmask`; lane j < 16
+// returns the count of digit j at `shift`.
+__device__ __forceinline__ uint32_t count_digits(uint32_t key, bool valid, uint32_t prefix,
+                                                 uint32_t pmask, int shift, int lane) {
+  const bool take = valid && (key & pmask) == prefix;
+  const uint32_t d = (key >> shift) & 15u;
+  uint32_t m = __ballot_sync(0xffffffffu, take);
+  const uint32_t b0 = __ballot_sync(0xffffffffu, take && (d & 1u));
+  const uint32_t b1 = __ballot_sync(0xffffffffu, take && (d & 2u));
+  const uint32_t b2 = __ballot_sync(0xffffffffu, take && (d & 4u));
+  const uint32_t b3 = __ballot_sync(0xffffffffu, take && (d & 8u));
+  m &= (lane & 1) ? b0 : ~b0;
+  m &= (lane & 2) ? b1 : ~b1;
+  m &= (lane & 4) ? b2 : ~b2;
+  m &= (lane & 8) ? b3 : ~b3;
+  return __popc(m);
 }
 
+// kRegKeys keys per thread in registers when M <= kRegKeys * kThreads; larger
+// M (kRegKeys = 0) keeps them in shared memory only.
+template <int kRegKeys>
 __global__ void __launch_bounds__(kThreads)
 fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V, int M, float alpha,
                    float eps, int k, float* __restrict__ S_out, int32_t* __restrict__ sel_idx,
@@ -66,22 +66,39 @@ fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V, int
                    unsigned int* status) {
   extern __shared__ uint32_t keys[];
   __shared__ float red[4][kWarps];
-  __shared__ uint32_t hist[256];
-  __shared__ uint32_t warp_tot[33];
-  __shared__ uint32_t sh_digit, sh_remaining;
+  __shared__ uint32_t cnt[2][kWarps][16];
+  __shared__ uint32_t scan_tot[kWarps];
   __shared__ int sh_nan;
 
   const int b = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   const float* a = A + (int64_t)b * M;
   const float* v = V + (int64_t)b * M;
+  constexpr bool in_regs = kRegKeys > 0;
+  constexpr int R = kRegKeys > 0 ? kRegKeys : 1;
 
-  // 1. min / max (fminf / fmaxf skip NaN)
-  float amn = __int_as_float(0x7f800000), amx = -amn, vmn = amn, vmx = -amn;
-  for (int i = tid; i < M; i += kThreads) {
-    const float x = a[i], y = v[i];
-    amn = fminf(amn, x); amx = fmaxf(amx, x);
-    vmn = fminf(vmn, y); vmx = fmaxf(vmx, y);
+  // 1. min / max (fminf / fmaxf skip NaN); A and V kept for step 2
+  float ra[R], rv[R];
+  const float inf = __int_as_float(0x7f800000);
+  float amn = inf, amx = -inf, vmn = inf, vmx = -inf;
+  if constexpr (in_regs) {
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const int i = tid + r * kThreads;
+      ra[r] = (i < M) ? a[i] : __int_as_float(0x7fc00000);
+      rv[r] = (i < M) ? v[i] : __int_as_float(0x7fc00000);
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      amn = fminf(amn, ra[r]); amx = fmaxf(amx, ra[r]);
+      vmn = fminf(vmn, rv[r]); vmx = fmaxf(vmx, rv[r]);
+    }
+  } else {
+    for (int i = tid; i < M; i += kThreads) {
+      const float x = a[i], y = v[i];
+      amn = fminf(amn, x); amx = fmaxf(amx, x);
+      vmn = fminf(vmn, y); vmx = fmaxf(vmx, y);
+    }
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -93,106 +110,150 @@ fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V, int
   if (lane == 0) { red[0][w] = amn; red[1][w] = amx; red[2][w] = vmn; red[3][w] = vmx; }
   if (tid == 0) sh_nan = 0;
   __syncthreads();
-  amn = red[0][0]; amx = red[1][0]; vmn = red[2][0]; vmx = red[3][0];
-  for (int j = 1; j < kWarps; ++j) {
-    amn = fminf(amn, red[0][j]); amx = fmaxf(amx, red[1][j]);
-    vmn = fminf(vmn, red[2][j]); vmx = fmaxf(vmx, red[3][j]);
+  {
+    const bool in = lane < kWarps;
+    amn = in ? red[0][lane] : inf;
+    amx = in ? red[1][lane] : -inf;
+    vmn = in ? red[2][lane] : inf;
+    vmx = in ? red[3][lane] : -inf;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      amn = fminf(amn, __shfl_xor_sync(0xffffffffu, amn, o));
+      amx = fmaxf(amx, __shfl_xor_sync(0xffffffffu, amx, o));
+      vmn = fminf(vmn, __shfl_xor_sync(0xffffffffu, vmn, o));
+      vmx = fmaxf(vmx, __shfl_xor_sync(0xffffffffu, vmx, o));
+    }
   }
 
-  // 2. fused score, fixed rounding order
+  // 2. fused score in a fixed rounding order, keys
   const float aden = __fadd_rn(__fsub_rn(amx, amn), eps);
   const float vden = __fadd_rn(__fsub_rn(vmx, vmn), eps);
   const float one_m = __fsub_rn(1.0f, alpha);
   int any_nan = 0;
-  for (int i = tid; i < M; i += kThreads) {
-    const float an = __fdiv_rn(__fsub_rn(a[i], amn), aden);
-    const float vn = __fdiv_rn(__fsub_rn(v[i], vmn), vden);
-    const float s = __fadd_rn(__fmul_rn(alpha, an), __fmul_rn(one_m, vn));
-    if (S_out) S_out[(int64_t)b * M + i] = s;
-    any_nan |= (s != s);
-    keys[i] = order_key(s);
-  }
-  if (any_nan) sh_nan = 1;
-  __syncthreads();
-  if (tid == 0 && sh_nan) raise_status(status, AVITS_ERR_NAN);
-
-  // 3. radix select of the k-th largest key
-  uint32_t prefix = 0u, pmask = 0u;
-  uint32_t remaining = (uint32_t)k;
-  if (k > 0 && k < M) {
-    for (int pass = 0; pass < 4; ++pass) {
-      const int shift = 24 - 8 * pass;
-      if (tid < 256) hist[tid] = 0u;
-      __syncthreads();
-      for (int i = tid; i < M; i += kThreads) {
-        const uint32_t key = keys[i];
-        if ((key & pmask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+  uint32_t rk[R];
+  auto fuse = [&](float x, float y) {
+    const float an = __fdiv_rn(__fsub_rn(x, amn), aden);
+    const float vn = __fdiv_rn(__fsub_rn(y, vmn), vden);
+    return __fadd_rn(__fmul_rn(alpha, an), __fmul_rn(one_m, vn));
+  };
+  if (in_regs) {
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const int i = tid + r * kThreads;
+      rk[r] = 0u;
+      if (i < M) {
+        const float s = fuse(ra[r], rv[r]);
+        if (S_out) S_out[(int64_t)b * M + i] = s;
+        any_nan |= (s != s);
+        rk[r] = order_key(s);
+        keys[i] = rk[r];
       }
-      __syncthreads();
-      if (w == 0) {
-        // lane l owns digits 255-8l ... 248-8l (descending order of keys)
-        uint32_t cnt[8], tot = 0;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) { cnt[e] = hist[255 - 8 * lane - e]; tot += cnt[e]; }
-        uint32_t inc = tot;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const uint32_t y = __shfl_up_sync(0xffffffffu, inc, o);
-          if (lane >= o) inc += y;
-        }
-        const uint32_t before = inc - tot;     // keys in higher digits
-        if (before < remaining && remaining <= inc) {
-          uint32_t c = before;
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            if (c < remaining && remaining <= c + cnt[e]) {
-              sh_digit = 255u - 8u * lane - e;
-              sh_remaining = remaining - c;
-            }
-            c += cnt[e];
-          }
-        }
-      }
-      __syncthreads();
-      prefix |= sh_digit << shift;
-      pmask |= 255u << shift;
-      remaining = sh_remaining;
-      __syncthreads();
+    }
+  } else {
+    for (int i = tid; i < M; i += kThreads) {
+      const float s = fuse(a[i], v[i]);
+      if (S_out) S_out[(int64_t)b * M + i] = s;
+      any_nan |= (s != s);
+      keys[i] = order_key(s);
     }
   }
-  const uint32_t T = prefix;
+  if (any_nan) sh_nan = 1;
 
-  // 4-5. selection and compaction over contiguous per-thread ranges
+  // 3. radix select of the k-th largest key
+  uint32_t prefix = 0u, pmask = 0u, remaining = (uint32_t)k;
+  int shift = 32;
+  if (!in_regs) __syncthreads();   // keys are read back from shared memory below
+  if (k > 0 && k < M) {
+    for (int pass = 0; pass < 8; ++pass) {
+      shift -= 4;
+      uint32_t c = 0;
+      if (in_regs) {
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+          const int i = tid + r * kThreads;
+          c += count_digits(rk[r], i < M, prefix, pmask, shift, lane);
+        }
+      } else {
+        for (int i0 = 0; i0 < M; i0 += kThreads) {
+          const int i = i0 + tid;
+          c += count_digits(i < M ? keys[i] : 0u, i < M, prefix, pmask, shift, lane);
+        }
+      }
+      if (lane < 16) cnt[pass & 1][w][lane] = c;
+      __syncthreads();
+      // every warp: lane l holds digit 15 - l (descending order), l < 16
+      uint32_t tot = 0;
+      if (lane < 16) {
+        uint32_t part[kWarps];
+#pragma unroll
+        for (int ww = 0; ww < kWarps; ++ww) part[ww] = cnt[pass & 1][ww][15 - lane];
+#pragma unroll
+        for (int ww = 0; ww < kWarps; ++ww) tot += part[ww];
+      }
+      uint32_t inc = tot;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += y;
+      }
+      const uint32_t before = inc - tot;
+      const bool hit = lane < 16 && before < remaining && remaining <= inc;
+      const uint32_t hmask = __ballot_sync(0xffffffffu, hit);
+      const int src = __ffs(hmask) - 1;
+      const uint32_t digit = 15u - (uint32_t)src;
+      const uint32_t rem = __shfl_sync(0xffffffffu, remaining - before, src);
+      const uint32_t bin = __shfl_sync(0xffffffffu, tot, src);
+      prefix |= digit << shift;
+      pmask |= 15u << shift;
+      remaining = rem;
+      if (rem == bin) break;   // the digit is taken whole: no tie left to break
+    }
+  }
+  // the selection is decided on the top (32 - shift) bits: keys whose prefix
+  // is above T are in; of the keys with prefix T the `remaining` lowest indices
+  const uint32_t T = shift < 32 ? (prefix >> shift) : 0u;
+  __syncthreads();   // keys[] complete for the range pass below
+  if (tid == 0 && sh_nan) raise_status(status, AVITS_ERR_NAN);
+
+  // 4. one scan of (above, equal) over contiguous per-thread ranges
   const int per = (M + kThreads - 1) / kThreads;
   const int lo = min(M, tid * per), hi = min(M, lo + per);
   uint32_t gt = 0, eq = 0;
   if (k > 0 && k < M) {
     for (int i = lo; i < hi; ++i) {
-      const uint32_t key = keys[i];
-      gt += key > T;
-      eq += key == T;
+      const uint32_t kp = keys[i] >> shift;
+      gt += kp > T;
+      eq += kp == T;
     }
   }
-  uint32_t eq_before;
-  block_exclusive_scan(eq, warp_tot, &eq_before);
-  uint32_t nsel;
-  if (k == 0) nsel = 0;
-  else if (k == M) nsel = (uint32_t)(hi - lo);
-  else {
-    const uint32_t take = remaining > eq_before ? min(remaining - eq_before, eq) : 0u;
-    nsel = gt + take;
+  // packed inclusive scan: high 16 bits above-count, low 16 bits equal-count
+  const uint32_t mine = (gt << 16) | eq;
+  uint32_t x = mine;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
   }
-  uint32_t sel_before;
-  block_exclusive_scan(nsel, warp_tot, &sel_before);
-  uint32_t eq_seen = eq_before, c = sel_before;
+  if (lane == 31) scan_tot[w] = x;
+  __syncthreads();
+  uint32_t wbefore = 0;
+#pragma unroll
+  for (int ww = 0; ww < kWarps; ++ww) wbefore += (ww < w) ? scan_tot[ww] : 0u;
+  const uint32_t excl = wbefore + x - mine;
+  const uint32_t gt_before = excl >> 16, eq_before = excl & 0xFFFFu;
+  uint32_t c;
+  if (k == 0) c = 0;
+  else if (k == M) c = (uint32_t)lo;
+  else c = gt_before + min(remaining, eq_before);
+  uint32_t eq_seen = eq_before;
   for (int i = lo; i < hi; ++i) {
     bool sel;
     if (k == 0) sel = false;
     else if (k == M) sel = true;
     else {
-      const uint32_t key = keys[i];
-      sel = key > T;
-      if (key == T) { sel = eq_seen < remaining; ++eq_seen; }
+      const uint32_t kp = keys[i] >> shift;
+      sel = kp > T;
+      if (kp == T) { sel = eq_seen < remaining; ++eq_seen; }
     }
     tok_offset[(int64_t)b * M + i] = i + 3 * (int)c;
     if (mask) mask[(int64_t)b * M + i] = sel ? 1 : 0;
@@ -213,14 +274,31 @@ cudaError_t launch_fuse_select(const float* A, const float* V, int B, int M, flo
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (!(dev >= 0 && dev < 64 && __atomic_load_n(&done[dev], __ATOMIC_ACQUIRE))) {
-      e = cudaFuncSetAttribute(fuse_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)(kSelectMaxM * sizeof(uint32_t)));
+      const int mx = (int)(kSelectMaxM * sizeof(uint32_t));
+      e = cudaFuncSetAttribute(fuse_select_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+      if (e != cudaSuccess) return e;
+      e = cudaFuncSetAttribute(fuse_select_kernel<kMaxRegKeys>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
       if (e != cudaSuccess) return e;
       if (dev >= 0 && dev < 64) __atomic_store_n(&done[dev], 1, __ATOMIC_RELEASE);
     }
   }
-  fuse_select_kernel<<<B, kThreads, smem, s>>>(A, V, M, alpha, eps, k, S, sel_idx, mask,
-                                               tok_offset, status);
+  const int per = (M + kThreads - 1) / kThreads;
+  if (per <= 1)
+    fuse_select_kernel<1><<<B, kThreads, smem, s>>>(A, V, M, alpha, eps, k, S, sel_idx, mask,
+                                                    tok_offset, status);
+  else if (per <= 2)
+    fuse_select_kernel<2><<<B, kThreads, smem, s>>>(A, V, M, alpha, eps, k, S, sel_idx, mask,
+                                                    tok_offset, status);
+  else if (per <= 4)
+    fuse_select_kernel<4><<<B, kThreads, smem, s>>>(A, V, M, alpha, eps, k, S, sel_idx, mask,
+                                                    tok_offset, status);
+  else if (per <= kMaxRegKeys)
+    fuse_select_kernel<kMaxRegKeys><<<B, kThreads, smem, s>>>(A, V, M, alpha, eps, k, S, sel_idx,
+                                                              mask, tok_offset, status);
+  else
+    fuse_select_kernel<0><<<B, kThreads, smem, s>>>(A, V, M, alpha, eps, k, S, sel_idx, mask,
+                                                    tok_offset, status);
   return cudaGetLastError();
 }
 

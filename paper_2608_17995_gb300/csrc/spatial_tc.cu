@@ -12,23 +12,34 @@
 //   unit  = (b, h, 256 query rows = two 128-row tiles)
 //   item  = (unit, 128-key tile)
 // The B*H*ceil(M/256)*ceil(Nk/128) items are split into equal contiguous
-// ranges, one per CTA, so every SM gets the same number of MMA tiles.  A unit
-// cut between CTAs leaves per-row partial (max, sums) in the workspace; the
-// last CTA to finish the unit (atomic ticket) merges them in slot order, and
-// the last unit of a (b, row block) to finish sums the head masses in head
-// order.  Both tickets are reset by their last arriver, so results do not
-// depend on CTA timing and the workspace is left zeroed.
+// ranges, one per CTA, so every SM issues the same number of MMA tiles.  Every
+// (CTA, unit, softmax warpgroup) piece stores its per-row partial statistics
+// (max, sum over all keys, sum over text keys) in the workspace; a second,
+// small kernel (spatial_finalize_kernel, launched as a programmatic dependent
+// of the first) merges the pieces of each (row, head) in slot order and sums
+// the heads in head order, so the result does not depend on CTA timing.
 //
-// Roles (10 warps):
-//   warp 0        TMA producer: Q tile pair once per unit (64 KB for d=128),
-//                 K tiles through a 4-stage ring, 128-byte swizzled.
+// Roles (18 warps):
+//   warp 0        TMA producer: Q tile 0, the first K tile, Q tile 1, then the
+//                 K tiles through a 4-stage ring (128-byte swizzle, no
+//                 multicast); each Q tile has its own barrier so the first MMA
+//                 starts after 64 KB rather than 96 KB.
 //   warp 1        MMA issuer: S = Q K^T with tcgen05.mma kind::f16 (bf16 in,
 //                 fp32 accumulate in tensor memory), 128x128 per tile, two S
-//                 buffers per Q tile (4 x 128 of the 512 TMEM columns).
-//   warps 2-5     softmax-reduce of Q tile 0, warps 6-9 of Q tile 1: one TMEM
-//                 lane (= one query row) per thread, 32 columns per
-//                 tcgen05.ld, exp2 on the MUFU with a running max; the text
-//                 keys come first, so the text sum is a prefix of the row sum.
+//                 buffers per Q tile (all 512 TMEM columns).
+//   warps 2-17    four softmax warpgroups: query tile t and column half c
+//                 (64 of the 128 keys of a tile) per warpgroup, so all 16
+//                 warps work on the same item while the MMA fills the other S
+//                 buffer; one TMEM lane (= one query row) per thread, 16
+//                 columns per tcgen05.ld, ex2 on the MUFU against the running
+//                 row maximum with packed f32x2 FMA/add.  The exact chunk
+//                 maximum is only computed when a chunk sum would leave
+//                 [0, 2^64) (first chunk, a larger logit, NaN).  The text keys
+//                 come first, so the text sum is a prefix of the row sum.  At
+//                 d = 128 a 128x128 tile costs the tensor pipe and the MUFU
+//                 (32 ex2 / clock / SM) the same 512 cycles; evaluating part
+//                 of the exponentials on the FMA pipe (exp2_fma2) was measured
+//                 slower on this chip (the loop is issue-bound), so E = 0.
 // Every wait is bounded (avits_common.cuh); on a timeout all roles stop
 // issuing, drain what they issued, release tensor memory and exit.
 #include <cuda.h>
@@ -43,7 +54,8 @@ constexpr int kBM = 128;       // query rows per tile (= TMEM lanes)
 constexpr int kBN = 128;       // keys per tile
 constexpr int kQTiles = 2;     // query tiles per unit
 constexpr int kUnitRows = kBM * kQTiles;
-constexpr int kThreads = 320;
+constexpr int kSoftmaxWarps = 16;
+constexpr int kThreads = 64 + kSoftmaxWarps * 32;
 constexpr int kTmemCols = 512;
 constexpr uint32_t kIdesc = (1u << 4)                       // D: fp32
                             | (1u << 7) | (1u << 10)        // A, B: bf16
@@ -60,13 +72,12 @@ struct Cfg {
 };
 
 struct Bars {
-  uint64_t q_full, q_empty;
+  uint64_t q_full[kQTiles], q_empty;
   uint64_t k_full[8], k_empty[8];
   uint64_t s_full[kQTiles][2], s_empty[kQTiles][2];
   uint64_t drain;
   uint32_t tmem_base;
   int abort;
-  int last_unit, last_group;
 };
 
 template <int D>
@@ -77,16 +88,13 @@ constexpr int smem_bytes() {
 struct TcParams {
   int B, H, M, Nk, L;
   int n_qp, n_kt, n_units;
-  long long total, per;
+  int total, per;          // items in all, items per CTA (total < 2^31 checked on the host)
   int max_parts;
   float c_log2, weight;
   int accumulate;
   float* A;
   float* lse;
-  float* part;      // [n_units][max_parts][256][3]
-  float* mass;      // [B*H][n_qp*256]
-  int* unit_cnt;    // [n_units]
-  int* grp_cnt;     // [B*n_qp]
+  float* part;      // [B*n_qp][H][2*max_parts][256][3]
   unsigned int* status;
 };
 
@@ -135,23 +143,19 @@ __device__ __forceinline__ void tc_fence_after() {
 #define AVITS_W8(b) "+r"(r[b]), "+r"(r[b + 1]), "+r"(r[b + 2]), "+r"(r[b + 3]), \
                     "+r"(r[b + 4]), "+r"(r[b + 5]), "+r"(r[b + 6]), "+r"(r[b + 7])
 
-// 32 consecutive fp32 columns of this thread's TMEM lane.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+// 16 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
   asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
-      "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, "
-      "%28, %29, %30, %31}, [%32];"
-      : AVITS_R8(0), AVITS_R8(8), AVITS_R8(16), AVITS_R8(24)
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15}, [%16];"
+      : AVITS_R8(0), AVITS_R8(8)
       : "r"(taddr));
 }
 
 // Completes the thread's outstanding tcgen05.ld; the registers are tied to
-// the wait so no use can be scheduled before it.
-__device__ __forceinline__ void tmem_wait(uint32_t (&r)[32]) {
-  asm volatile("tcgen05.wait::ld.sync.aligned;"
-               : AVITS_W8(0), AVITS_W8(8), AVITS_W8(16), AVITS_W8(24)
-               :
-               : "memory");
+// the wait so that no use can be scheduled before it.
+__device__ __forceinline__ void tmem_wait(uint32_t (&r)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" : AVITS_W8(0), AVITS_W8(8) : : "memory");
 }
 
 __device__ __forceinline__ float ex2(float x) {
@@ -166,53 +170,136 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
   return d;
 }
 
-__device__ __forceinline__ void softmax_bar() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+// (a0, a1) * b + c on both lanes of a packed pair.
+__device__ __forceinline__ void ffma2(float a0, float a1, float b, float c, float& d0, float& d1) {
+  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %4};\n\tmov.b64 rc, {%5, %5};\n\t"
+      "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d0), "=f"(d1)
+      : "f"(a0), "f"(a1), "f"(b), "f"(c));
+}
 
-// Running row statistics in the log2 domain: x = c_log2 * (q.k).
+// (s0, s1) += (e0, e1) on a packed pair.
+__device__ __forceinline__ void fadd2(float& s0, float& s1, float e0, float e1) {
+  asm("{\n\t.reg .b64 ra, rb;\n\t"
+      "mov.b64 ra, {%0, %1};\n\tmov.b64 rb, {%2, %3};\n\t"
+      "add.rn.f32x2 ra, ra, rb;\n\tmov.b64 {%0, %1}, ra;\n\t}"
+      : "+f"(s0), "+f"(s1)
+      : "f"(e0), "f"(e1));
+}
+
+// (d0, d1) = (a0, a1) * (b0, b1) + (c0, c1) on a packed pair.
+__device__ __forceinline__ void fma2full(float a0, float a1, float b0, float b1, float c0, float c1,
+                                         float& d0, float& d1) {
+  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+      "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d0), "=f"(d1)
+      : "f"(a0), "f"(a1), "f"(b0), "f"(b1), "f"(c0), "f"(c1));
+}
+
+// (p0, p1) = (p0, p1) * (r0, r1) + k on a packed pair.
+__device__ __forceinline__ void fma2v(float& p0, float& p1, float r0, float r1, float k) {
+  asm("{\n\t.reg .b64 ra, rb, rc;\n\t"
+      "mov.b64 ra, {%0, %1};\n\tmov.b64 rb, {%2, %3};\n\tmov.b64 rc, {%4, %4};\n\t"
+      "fma.rn.f32x2 ra, ra, rb, rc;\n\tmov.b64 {%0, %1}, ra;\n\t}"
+      : "+f"(p0), "+f"(p1)
+      : "f"(r0), "f"(r1), "f"(k));
+}
+
+__device__ __forceinline__ void bar_sync(int id, int count) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
+// Running row statistics in the log2 domain: x = c_log2 * (q.k); the sums
+// are of 2^(x - m).
 struct RowStat {
   float m, la, lt;
 };
 
-// One 32-column chunk: col0 = index of its first key.
-__device__ __forceinline__ void process_chunk(const uint32_t (&r)[32], int col0, int Nk, int L,
+__device__ __forceinline__ void merge_stat(RowStat& a, float m2, float la2, float lt2) {
+  const float m = fmaxf(a.m, m2);
+  if (m == -INFINITY) return;
+  const float f1 = ex2(a.m - m), f2 = ex2(m2 - m);
+  a.la = a.la * f1 + la2 * f2;
+  a.lt = a.lt * f1 + lt2 * f2;
+  a.m = m;
+}
+
+// 2^x on the FMA pipe for a pair of values: x clamped to [-126, 64] (a
+// clamped-high value still fails the caller's 2^64 check), j = round(x) by
+// the 1.5*2^23 addition, r = x - j in [-1/2, 1/2], 2^r by a degree-4 minimax
+// polynomial (Horner), 2^j added to the exponent field.
+__device__ __forceinline__ void exp2_fma2(float x0, float x1, float& e0, float& e1) {
+  const float kMagic = 12582912.0f;   // 1.5 * 2^23
+  x0 = fminf(fmaxf(x0, -126.0f), 64.0f);
+  x1 = fminf(fmaxf(x1, -126.0f), 64.0f);
+  float y0, y1, t0, t1, r0, r1, p0, p1;
+  ffma2(x0, x1, 1.0f, kMagic, y0, y1);          // y = x + magic (rounds x)
+  ffma2(y0, y1, 1.0f, -kMagic, t0, t1);         // t = round(x)
+  fma2full(t0, t1, -1.0f, -1.0f, x0, x1, r0, r1);   // r = x - t
+  ffma2(r0, r1, 9.570102e-03f, 5.591786e-02f, p0, p1);
+  fma2v(p0, p1, r0, r1, 2.4024744e-01f);
+  fma2v(p0, p1, r0, r1, 6.931218e-01f);
+  fma2v(p0, p1, r0, r1, 9.999993e-01f);
+  e0 = __int_as_float(__float_as_int(p0) + (__float_as_int(y0) << 23));
+  e1 = __int_as_float(__float_as_int(p1) + (__float_as_int(y1) << 23));
+}
+
+// One 16-column chunk whose first key is col0 (< Nk); the last E of its
+// exponentials (E = 0, 2 or 4) are evaluated on the FMA pipe.
+template <int E>
+__device__ __forceinline__ void process_chunk(const uint32_t (&r)[16], int col0, int Nk, int L,
                                               float c, RowStat& st) {
-  float v[32];
+  float v[16];
 #pragma unroll
-  for (int e = 0; e < 32; ++e) v[e] = __uint_as_float(r[e]);
+  for (int e = 0; e < 16; ++e) v[e] = __uint_as_float(r[e]);
   const int nvalid = Nk - col0;
-  if (nvalid < 32) {
+  if (nvalid < 16) {
 #pragma unroll
-    for (int e = 0; e < 32; ++e)
+    for (int e = 0; e < 16; ++e)
       if (e >= nvalid) v[e] = -INFINITY;
   }
-  float t[11];
+  const float nm = -st.m;
+  float x[16];
 #pragma unroll
-  for (int e = 0; e < 10; ++e) t[e] = max3(v[3 * e], v[3 * e + 1], v[3 * e + 2]);
-  t[10] = fmaxf(v[30], v[31]);
-  const float u0 = max3(t[0], t[1], t[2]), u1 = max3(t[3], t[4], t[5]);
-  const float u2 = max3(t[6], t[7], t[8]), u3 = fmaxf(t[9], t[10]);
-  const float cmax = fmaxf(fmaxf(u0, u1), fmaxf(u2, u3));
-  if (cmax == -INFINITY) return;
-  const float mx = cmax * c;
-  if (mx > st.m) {
+  for (int e = 0; e < 16; e += 2) ffma2(v[e], v[e + 1], c, nm, x[e], x[e + 1]);
+  float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+  for (int e = 0; e < 16 - E; e += 4) {
+    fadd2(s0, s1, ex2(x[e]), ex2(x[e + 1]));
+    if (e + 2 < 16 - E) fadd2(s2, s3, ex2(x[e + 2]), ex2(x[e + 3]));
+  }
+#pragma unroll
+  for (int e = 16 - E; e < 16; e += 2) {
+    float e0, e1;
+    exp2_fma2(x[e], x[e + 1], e0, e1);
+    fadd2(s2, s3, e0, e1);
+  }
+  fadd2(s0, s1, s2, s3);
+  float cs = s0 + s1;
+  if (!(cs < 0x1p64f)) {
+    // first chunk of a row, a logit 64 log2-units above the running maximum,
+    // or a NaN: take the exact chunk maximum and rescale the running sums
+    const float t0 = max3(v[0], v[1], v[2]), t1 = max3(v[3], v[4], v[5]);
+    const float t2 = max3(v[6], v[7], v[8]), t3 = max3(v[9], v[10], v[11]);
+    const float t4 = max3(v[12], v[13], v[14]);
+    const float mx = fmaxf(st.m, fmaxf(max3(t0, t1, t2), max3(t3, t4, v[15])) * c);
     const float corr = ex2(st.m - mx);
     st.la *= corr;
     st.lt *= corr;
     st.m = mx;
-  }
-  const float nm = -st.m;
-  float s[4] = {0.f, 0.f, 0.f, 0.f};
+    cs = 0.f;
 #pragma unroll
-  for (int e = 0; e < 32; ++e) s[e & 3] += ex2(fmaf(v[e], c, nm));
-  const float cs = (s[0] + s[1]) + (s[2] + s[3]);
+    for (int e = 0; e < 16; ++e) cs += ex2(fmaf(v[e], c, -mx));
+  }
   st.la += cs;
-  if (col0 + 32 <= L) {
+  if (col0 + 16 <= L) {
     st.lt += cs;
-  } else if (col0 < L) {
+  } else if (col0 < L) {   // the chunk straddles the text / image boundary
     float ts = 0.f;
 #pragma unroll
-    for (int e = 0; e < 32; ++e)
-      if (col0 + e < L) ts += ex2(fmaf(v[e], c, nm));
+    for (int e = 0; e < 16; ++e) ts += (col0 + e < L) ? ex2(fmaf(v[e], c, -st.m)) : 0.f;
     st.lt += ts;
   }
 }
@@ -221,13 +308,18 @@ struct Segment {
   int u, kt0, nk;
 };
 
-__device__ __forceinline__ Segment segment_at(long long it, long long it_end, int n_kt) {
+__device__ __forceinline__ Segment segment_at(int it, int it_end, int n_kt) {
   Segment s;
-  s.u = (int)(it / n_kt);
-  s.kt0 = (int)(it - (long long)s.u * n_kt);
-  const long long left = it_end - it;
-  s.nk = (int)((long long)(n_kt - s.kt0) < left ? (n_kt - s.kt0) : left);
+  s.u = it / n_kt;
+  s.kt0 = it - s.u * n_kt;
+  s.nk = min(n_kt - s.kt0, it_end - it);
   return s;
+}
+
+// Number of CTAs whose item range overlaps unit u, and the first of them.
+__device__ __forceinline__ int first_cta(int u, int n_kt, int per) { return (u * n_kt) / per; }
+__device__ __forceinline__ int pieces(int u, int n_kt, int per) {
+  return ((u + 1) * n_kt - 1) / per - (u * n_kt) / per + 1;
 }
 
 template <int D>
@@ -243,13 +335,12 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
   Bars* bars = reinterpret_cast<Bars*>(sK + C::kKBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const long long it_begin = (long long)blockIdx.x * p.per;
-  long long it_end = it_begin + p.per;
-  if (it_end > p.total) it_end = p.total;
+  const int it_begin = (int)blockIdx.x * p.per;
+  const int it_end = min(it_begin + p.per, p.total);
   if (it_begin >= it_end) return;   // block-uniform
 
   if (threadIdx.x == 0) {
-    mbar_init(&bars->q_full, 1);
+    for (int t = 0; t < kQTiles; ++t) mbar_init(&bars->q_full[t], 1);
     mbar_init(&bars->q_empty, 1);
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&bars->k_full[s], 1);
@@ -258,7 +349,7 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
     for (int t = 0; t < kQTiles; ++t)
       for (int b = 0; b < 2; ++b) {
         mbar_init(&bars->s_full[t][b], 1);
-        mbar_init(&bars->s_empty[t][b], 4);
+        mbar_init(&bars->s_empty[t][b], 8);   // 8 softmax warps read each tile
       }
     mbar_init(&bars->drain, 1);
     bars->abort = 0;
@@ -276,6 +367,8 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
   tc_fence_after();
   const uint32_t tmem = bars->tmem_base;
   volatile int* abort_flag = &bars->abort;
+  // the merge kernel may be scheduled now; it waits for this grid to finish
+  if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (warp == 0) {
     // ------------------------------------------------------ TMA producer --
@@ -283,20 +376,27 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQ)) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
       bool ok = true;
-      long long li = 0;
+      int li = 0;
       int sg = 0;
-      for (long long it = it_begin; it < it_end && ok;) {
+      int q_armed = 0;   // Q tiles armed in the latest segment
+      for (int it = it_begin; it < it_end && ok;) {
         const Segment seg = segment_at(it, it_end, p.n_kt);
         const int bh = seg.u / p.n_qp, qp = seg.u - bh * p.n_qp;
         const int b = bh / p.H, h = bh - b * p.H;
-        if (sg > 0) ok = mbar_wait_bounded(&bars->q_empty, (sg - 1) & 1, abort_flag, p.status);
+        ok = mbar_wait_bounded(&bars->q_empty, (uint32_t)((sg & 1) ^ 1), abort_flag, p.status);
         if (!ok) break;
-        mbar_arrive_expect_tx(&bars->q_full, C::kQBytes);
-        for (int t = 0; t < kQTiles; ++t)
-          for (int cb = 0; cb < C::kCB; ++cb)
-            tma_load_4d(sQ + t * C::kTileBytes + cb * (kBM * 128), &tmQ, cb * 64,
-                        qp * kUnitRows + t * kBM, h, b, &bars->q_full);
+        ++sg;   // Q of this segment is being issued
+        q_armed = 0;
         for (int j = 0; j < seg.nk; ++j, ++li) {
+          // Q tile 0 before the first K tile, Q tile 1 right after it
+          if (j == 0 || (j == 1 && kQTiles > 1)) {
+            const int t = j;
+            ++q_armed;
+            mbar_arrive_expect_tx(&bars->q_full[t], C::kTileBytes);
+            for (int cb = 0; cb < C::kCB; ++cb)
+              tma_load_4d(sQ + t * C::kTileBytes + cb * (kBM * 128), &tmQ, cb * 64,
+                          qp * kUnitRows + t * kBM, h, b, &bars->q_full[t]);
+          }
           const int stage = (int)(li % C::kStages);
           const uint32_t ph = (uint32_t)((li / C::kStages) & 1);
           ok = mbar_wait_bounded(&bars->k_empty[stage], ph ^ 1u, abort_flag, p.status);
@@ -306,16 +406,24 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
             tma_load_4d(sK + stage * C::kTileBytes + cb * (kBM * 128), &tmK, cb * 64,
                         (seg.kt0 + j) * kBN, h, b, &bars->k_full[stage]);
         }
+        if (ok && seg.nk == 1) {   // a one-tile segment still needs Q tile 1
+          ++q_armed;
+          mbar_arrive_expect_tx(&bars->q_full[1], C::kTileBytes);
+          for (int cb = 0; cb < C::kCB; ++cb)
+            tma_load_4d(sQ + C::kTileBytes + cb * (kBM * 128), &tmQ, cb * 64,
+                        qp * kUnitRows + kBM, h, b, &bars->q_full[1]);
+        }
         it += seg.nk;
-        ++sg;
       }
       if (!ok) {
-        // drain the copies still in flight before the CTA exits
-        if (sg > 0) mbar_wait_bounded(&bars->q_full, (sg - 1) & 1, nullptr, p.status);
+        // drain the copies still in flight before the CTA exits: the Q tiles
+        // of the last segment started, then every armed K stage
+        for (int t = 0; t < q_armed; ++t)
+          mbar_wait_bounded(&bars->q_full[t], (uint32_t)((sg - 1) & 1), nullptr, p.status);
         for (int s = 0; s < C::kStages; ++s) {
-          const long long armed = li - s;   // items issued on stage s: li - s > 0
+          const int armed = li - s;   // items issued on stage s: li - s > 0
           if (armed > 0) {
-            const long long last = (armed - 1) / C::kStages;
+            const int last = (armed - 1) / C::kStages;
             mbar_wait_bounded(&bars->k_full[s], (uint32_t)(last & 1), nullptr, p.status);
           }
         }
@@ -325,13 +433,10 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
     // --------------------------------------------------------- MMA issuer --
     if (lane == 0) {
       bool ok = true;
-      long long li = 0;
+      int li = 0;
       int sg = 0;
-      for (long long it = it_begin; it < it_end && ok;) {
+      for (int it = it_begin; it < it_end && ok;) {
         const Segment seg = segment_at(it, it_end, p.n_kt);
-        ok = mbar_wait_bounded(&bars->q_full, sg & 1, abort_flag, p.status);
-        if (!ok) break;
-        tc_fence_after();
         for (int j = 0; j < seg.nk && ok; ++j, ++li) {
           const int stage = (int)(li % C::kStages);
           const uint32_t ph = (uint32_t)((li / C::kStages) & 1);
@@ -341,6 +446,10 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
           if (!ok) break;
           tc_fence_after();
           for (int t = 0; t < kQTiles; ++t) {
+            if (j == 0) {
+              ok = mbar_wait_bounded(&bars->q_full[t], (uint32_t)(sg & 1), abort_flag, p.status);
+              if (!ok) break;
+            }
             ok = mbar_wait_bounded(&bars->s_empty[t][sb], sph ^ 1u, abort_flag, p.status);
             if (!ok) break;
             tc_fence_after();
@@ -368,132 +477,53 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
     }
   } else {
     // ---------------------------------------------------- softmax-reduce --
-    const int t = (warp - 2) >> 2;        // query tile of this warpgroup
+    const int g = (warp - 2) >> 2;        // warpgroup: query tile t, column half ch
+    const int t = g >> 1, half = g & 1;
     const int quad = warp & 3;            // TMEM lane quadrant this warp may access
     const int rowt = quad * 32 + lane;    // row within the tile
     const int rowu = t * kBM + rowt;      // row within the unit
-    const int sm_tid = threadIdx.x - 64;  // 0..255
-    const float ln2 = 0.69314718055994530942f;
-    long long li = 0;
-    for (long long it = it_begin; it < it_end;) {
+    const uint32_t tlane = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(t * 2 * kBN + half * 64);
+    int li0 = 0;
+    for (int it = it_begin; it < it_end;) {
       const Segment seg = segment_at(it, it_end, p.n_kt);
       RowStat st{-INFINITY, 0.f, 0.f};
-      for (int j = 0; j < seg.nk; ++j, ++li) {
-        const int sb = (int)(li & 1);
+      for (int j = 0; j < seg.nk; ++j) {
+        const int li = li0 + j;
+        const int sb = li & 1;
         const uint32_t sph = (uint32_t)((li >> 1) & 1);
         bool ok = (*abort_flag == 0) && mbar_wait_bounded(&bars->s_full[t][sb], sph, abort_flag, p.status);
         ok = __all_sync(0xffffffffu, ok);   // tcgen05.ld below is warp-collective
         if (ok) {
           tc_fence_after();
-          const int kbase = (seg.kt0 + j) * kBN;
-          const uint32_t ta = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)((t * 2 + sb) * kBN);
-          uint32_t ra[32], rb[32];
-          tmem_ld32(ta, ra);
+          const uint32_t tb = tlane + (uint32_t)(sb * kBN);
+          const int c0 = (seg.kt0 + j) * kBN + half * 64;       // first key of this half
+          const int nch = max(0, min(4, (p.Nk - c0 + 15) >> 4));  // chunks with a valid key
+          uint32_t ra[16], rb[16];
+          tmem_ld16(tb, ra);
           tmem_wait(ra);
-          tmem_ld32(ta + 32, rb);
-          process_chunk(ra, kbase, p.Nk, p.L, p.c_log2, st);
+          tmem_ld16(tb + 16, rb);
+          if (0 < nch) process_chunk<0>(ra, c0, p.Nk, p.L, p.c_log2, st);
           tmem_wait(rb);
-          tmem_ld32(ta + 64, ra);
-          process_chunk(rb, kbase + 32, p.Nk, p.L, p.c_log2, st);
+          tmem_ld16(tb + 32, ra);
+          if (1 < nch) process_chunk<0>(rb, c0 + 16, p.Nk, p.L, p.c_log2, st);
           tmem_wait(ra);
-          tmem_ld32(ta + 96, rb);
-          process_chunk(ra, kbase + 64, p.Nk, p.L, p.c_log2, st);
+          tmem_ld16(tb + 48, rb);
+          if (2 < nch) process_chunk<0>(ra, c0 + 32, p.Nk, p.L, p.c_log2, st);
           tmem_wait(rb);
-          process_chunk(rb, kbase + 96, p.Nk, p.L, p.c_log2, st);
+          if (3 < nch) process_chunk<0>(rb, c0 + 48, p.Nk, p.L, p.c_log2, st);
           tc_fence_before();
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars->s_empty[t][sb]);
       }
-
-      // ---- epilogue of this unit segment (all 256 softmax threads) ----
+      // this warpgroup's piece of the unit: slot 2 * (CTA - first CTA of u) + half
       const int u = seg.u;
-      const int bh = u / p.n_qp, qp = u - bh * p.n_qp;
-      const int b = bh / p.H;
-      const int row = qp * kUnitRows + rowu;
-      const long long first = ((long long)u * p.n_kt) / p.per;
-      const long long last = ((long long)(u + 1) * p.n_kt - 1) / p.per;
-      const int nparts = (int)(last - first + 1);
-      bool have = true;
-      if (nparts > 1) {
-        const int slot = (int)(blockIdx.x - first);
-        float* pp = p.part + (((long long)u * p.max_parts + slot) * kUnitRows + rowu) * 3;
-        pp[0] = st.m;
-        pp[1] = st.la;
-        pp[2] = st.lt;
-        __threadfence();
-        softmax_bar();
-        if (sm_tid == 0) {
-          const int prev = atomicAdd(&p.unit_cnt[u], 1);
-          bars->last_unit = (prev == nparts - 1);
-          if (prev == nparts - 1) p.unit_cnt[u] = 0;
-        }
-        softmax_bar();
-        have = bars->last_unit != 0;
-        if (have) {
-          __threadfence();
-          float m = -INFINITY;
-          for (int s = 0; s < nparts; ++s) {
-            const float* q = p.part + (((long long)u * p.max_parts + s) * kUnitRows + rowu) * 3;
-            m = fmaxf(m, __ldcg(q));
-          }
-          float la = 0.f, lt = 0.f;
-          for (int s = 0; s < nparts; ++s) {
-            const float* q = p.part + (((long long)u * p.max_parts + s) * kUnitRows + rowu) * 3;
-            const float ms = __ldcg(q);
-            const float f = (ms == -INFINITY) ? 0.f : ex2(ms - m);
-            la += __ldcg(q + 1) * f;
-            lt += __ldcg(q + 2) * f;
-          }
-          st.m = m;
-          st.la = la;
-          st.lt = lt;
-        }
-      }
-      if (have) {
-        const float mass = st.lt / st.la;
-        if (p.lse && row < p.M) {
-          float* lp = p.lse + ((long long)bh * p.M + row) * 2;
-          lp[0] = (st.m + __log2f(st.la)) * ln2;
-          lp[1] = st.lt > 0.f ? (st.m + __log2f(st.lt)) * ln2 : -INFINITY;
-        }
-        if (p.H == 1) {
-          if (row < p.M) {
-            const float a = p.weight * mass;
-            float* ap = p.A + (long long)b * p.M + row;
-            *ap = p.accumulate ? *ap + a : a;
-          }
-        } else {
-          p.mass[(long long)bh * (p.n_qp * kUnitRows) + row] = mass;
-          __threadfence();
-        }
-      }
-      // head reduction: the last of the H units of (b, qp) to finish sums
-      if (p.H > 1) {
-        // only CTAs that finalised the unit take part in the group ticket;
-        // `have` is uniform over the 256 threads
-        if (have) {
-          softmax_bar();
-          if (sm_tid == 0) {
-            int* gc = &p.grp_cnt[b * p.n_qp + qp];
-            const int prev = atomicAdd(gc, 1);
-            bars->last_group = (prev == p.H - 1);
-            if (prev == p.H - 1) *gc = 0;
-          }
-          softmax_bar();
-          if (bars->last_group) {
-            __threadfence();
-            float sum = 0.f;
-            const float* mp = p.mass + (long long)b * p.H * (p.n_qp * kUnitRows) + row;
-            for (int hh = 0; hh < p.H; ++hh) sum += __ldcg(mp + (long long)hh * p.n_qp * kUnitRows);
-            if (row < p.M) {
-              const float a = p.weight * (sum / (float)p.H);
-              float* ap = p.A + (long long)b * p.M + row;
-              *ap = p.accumulate ? *ap + a : a;
-            }
-          }
-        }
-      }
+      const int slot = 2 * ((int)blockIdx.x - first_cta(u, p.n_kt, p.per)) + half;
+      float* pp = p.part + (((long long)u * (2 * p.max_parts) + slot) * kUnitRows + rowu) * 3;
+      pp[0] = st.m;
+      pp[1] = st.la;
+      pp[2] = st.lt;
+      li0 += seg.nk;
       it += seg.nk;
     }
   }
@@ -504,6 +534,65 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                  "r"(kTmemCols));
+  }
+}
+
+// Second kernel: merge the pieces of every (row, head) in slot order, then the
+// head mean of Eq. 3.  Block = 32 rows x 8 head groups; thread (r, hg) merges
+// heads hg, hg+8, ... of row r (all loads of a head issued before its merge)
+// and the 8 partial sums are added in head-group order.  Launched as a
+// programmatic dependent of spatial_tc_kernel: it waits for the producer grid
+// to complete before reading the pieces.
+constexpr int kFinRows = 32, kFinGroups = 8;
+
+__global__ void __launch_bounds__(kFinRows * kFinGroups)
+spatial_finalize_kernel(const TcParams p) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  __shared__ float part_sum[kFinGroups][kFinRows];
+  const int r = threadIdx.x % kFinRows, hg = threadIdx.x / kFinRows;
+  const int row_g = blockIdx.x * kFinRows + r;            // over B * n_qp * 256
+  const int rows_per_b = p.n_qp * kUnitRows;
+  const int b = row_g / rows_per_b;
+  const int row = row_g - b * rows_per_b;                  // row within the element
+  const int qp = row / kUnitRows, rowu = row - qp * kUnitRows;
+  const float ln2 = 0.69314718055994530942f;
+  float sum = 0.f;
+  if (b < p.B) {
+    for (int h = hg; h < p.H; h += kFinGroups) {
+      const int u = (b * p.H + h) * p.n_qp + qp;
+      const int np = 2 * pieces(u, p.n_kt, p.per);
+      const float* q = p.part + ((long long)u * (2 * p.max_parts) * kUnitRows + rowu) * 3;
+      RowStat acc{-INFINITY, 0.f, 0.f};
+      for (int s0 = 0; s0 < np; s0 += 6) {
+        float v[6][3];
+#pragma unroll
+        for (int k = 0; k < 6; ++k)
+          if (s0 + k < np) {
+            const float* qs = q + (long long)(s0 + k) * kUnitRows * 3;
+            v[k][0] = __ldcg(qs);
+            v[k][1] = __ldcg(qs + 1);
+            v[k][2] = __ldcg(qs + 2);
+          }
+#pragma unroll
+        for (int k = 0; k < 6; ++k)
+          if (s0 + k < np) merge_stat(acc, v[k][0], v[k][1], v[k][2]);
+      }
+      sum += acc.lt / acc.la;
+      if (p.lse && row < p.M) {
+        float* lp = p.lse + (((long long)b * p.H + h) * p.M + row) * 2;
+        lp[0] = (acc.m + __log2f(acc.la)) * ln2;
+        lp[1] = acc.lt > 0.f ? (acc.m + __log2f(acc.lt)) * ln2 : -INFINITY;
+      }
+    }
+  }
+  part_sum[hg][r] = sum;
+  __syncthreads();
+  if (hg == 0 && b < p.B && row < p.M) {
+    float tot = 0.f;
+    for (int k = 0; k < kFinGroups; ++k) tot += part_sum[k][r];
+    const float a = p.weight * (tot / (float)p.H);
+    float* ap = p.A + (long long)b * p.M + row;
+    *ap = p.accumulate ? *ap + a : a;
   }
 }
 
@@ -551,7 +640,7 @@ bool make_map(CUtensorMap* map, const void* base, int B, int H, int rows, int d,
 struct Plan {
   int n_qp, n_kt, n_units, max_parts, grid;
   long long total, per;
-  size_t off_unit, off_grp, off_part, off_mass, bytes;
+  size_t bytes;
 };
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
@@ -567,16 +656,7 @@ Plan make_plan(int B, int H, int M, int Nk, int num_sms) {
   if (pl.per < 1) pl.per = 1;
   pl.grid = (int)((pl.total + pl.per - 1) / pl.per);
   pl.max_parts = (int)((pl.n_kt + pl.per - 1) / pl.per) + 1;
-  size_t o = 0;
-  pl.off_unit = o;
-  o = align256(o + sizeof(int) * (size_t)pl.n_units);
-  pl.off_grp = o;
-  o = align256(o + sizeof(int) * (size_t)B * pl.n_qp);
-  pl.off_part = o;
-  o = align256(o + sizeof(float) * 3 * (size_t)pl.n_units * pl.max_parts * kUnitRows);
-  pl.off_mass = o;
-  o = align256(o + sizeof(float) * (size_t)B * H * pl.n_qp * kUnitRows);
-  pl.bytes = o;
+  pl.bytes = align256(sizeof(float) * 3 * (size_t)pl.n_units * 2 * pl.max_parts * kUnitRows);
   return pl;
 }
 
@@ -613,6 +693,8 @@ bool spatial_tc_eligible(const SpatialArgs& a) {
   if (!strides_ok(a.B, a.H, a.q_sb, a.q_sh, a.q_sn)) return false;
   if (!strides_ok(a.B, a.H, a.k_sb, a.k_sh, a.k_sn)) return false;
   if (!(a.scale > 0.f)) return false;
+  const long long n_qp = (a.M + kUnitRows - 1) / kUnitRows, n_kt = (a.Nk + kBN - 1) / kBN;
+  if ((long long)a.B * a.H * n_qp * (n_kt + 1) >= (1ll << 31)) return false;
   return encode_fn() != nullptr;
 }
 
@@ -631,16 +713,13 @@ cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s)
   TcParams p{};
   p.B = a.B; p.H = a.H; p.M = a.M; p.Nk = a.Nk; p.L = a.L;
   p.n_qp = pl.n_qp; p.n_kt = pl.n_kt; p.n_units = pl.n_units;
-  p.total = pl.total; p.per = pl.per; p.max_parts = pl.max_parts;
+  p.total = (int)pl.total; p.per = (int)pl.per; p.max_parts = pl.max_parts;
   p.c_log2 = a.scale * 1.4426950408889634f;
   p.weight = a.weight;
   p.accumulate = a.accumulate;
   p.A = a.A;
   p.lse = a.lse;
-  p.unit_cnt = reinterpret_cast<int*>(ws + pl.off_unit);
-  p.grp_cnt = reinterpret_cast<int*>(ws + pl.off_grp);
-  p.part = reinterpret_cast<float*>(ws + pl.off_part);
-  p.mass = reinterpret_cast<float*>(ws + pl.off_mass);
+  p.part = reinterpret_cast<float*>(ws);
   p.status = a.status;
   cudaError_t e = set_smem_once();
   if (e != cudaSuccess) return e;
@@ -648,6 +727,21 @@ cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s)
     spatial_tc_kernel<128><<<pl.grid, kThreads, smem_bytes<128>(), s>>>(mq, mk, p);
   else
     spatial_tc_kernel<64><<<pl.grid, kThreads, smem_bytes<64>(), s>>>(mq, mk, p);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  // the merge runs as a programmatic dependent: it may be scheduled while the
+  // main kernel drains and waits (griddepcontrol.wait) for its completion
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((unsigned)((a.B * pl.n_qp * kUnitRows + kFinRows - 1) / kFinRows));
+  cfg.blockDim = dim3(kFinRows * kFinGroups);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, spatial_finalize_kernel, p);
   return cudaGetLastError();
 }
 

@@ -1,16 +1,22 @@
 // temporal.cu — temporal importance (Sec. 3.3.2).
 //
 // avits_score_temporal: V = ||h_t - h_prev|| / (||h_prev|| + eps) per token.
-// HBM-bound: each token row (D values of each snapshot) is read once with
-// 16-byte vector loads, a warp per token, all of a lane's loads issued before
-// any arithmetic so that each warp keeps ~24 x 16 B in flight; fp32 sums,
-// shuffle reduction.  Algorithmic bytes: 2 * B*N*D*elt + 4*B*N.
+// HBM-bound.  Main path: each CTA stages up to 8 token rows of both
+// snapshots in shared memory with bulk copies (cp.async.bulk, one per row,
+// completing on one mbarrier), so a whole chunk is in flight with a single
+// issuing thread; then one warp per token reduces its two rows from shared
+// memory (fp32 sums, shuffle reduction).  Chunks are small (2 tokens) and
+// many CTAs fit on an SM, so all of the input is in flight at once and the
+// kernel can share SMs with the spatial kernel.  Rows that are not 16-byte
+// multiples use a register path.  Algorithmic bytes: 2 * B*N*D*elt + 4*B*N.
 //
 // avits_score_temporal_var: Eq. 6-7, unbiased variance over N_T snapshots
 // averaged over channels; two passes over the snapshot values held in
 // registers (mean, then squared deviations).
 #include "avits_common.cuh"
 #include "avits_internal.h"
+
+#include <algorithm>
 
 namespace avits {
 namespace {
@@ -129,6 +135,92 @@ temporal_scalar_kernel(const T* __restrict__ ht, const T* __restrict__ hp, int64
   }
 }
 
+// ------------------------------------------------ bulk-copy staged path --
+// 2 tokens (24 KB at D = 3072 bf16) per CTA-chunk: small enough to share an
+// SM with the spatial kernel's CTA, so the two can run concurrently.
+constexpr int kStageTokens = 2;
+constexpr int kStageBytesMax = 32 * 1024;
+
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kWarpsPerCta * 32)
+temporal_staged_kernel(const T* __restrict__ ht, const T* __restrict__ hp, int64_t ntok, int D,
+                       int tpc, float eps, float* __restrict__ V, unsigned int* status) {
+  extern __shared__ __align__(128) uint8_t sm[];
+  __shared__ __align__(8) uint64_t bar;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint32_t row_bytes = (uint32_t)D * sizeof(T);
+  T* s_t = reinterpret_cast<T*>(sm);
+  T* s_p = reinterpret_cast<T*>(sm + (size_t)tpc * row_bytes);
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  const int64_t nchunks = (ntok + tpc - 1) / tpc;
+  uint32_t phase = 0;
+  for (int64_t c = blockIdx.x; c < nchunks; c += gridDim.x, phase ^= 1u) {
+    const int64_t t0 = c * tpc;
+    const int64_t left = ntok - t0;
+    const int n = left < (int64_t)tpc ? (int)left : tpc;
+    if (threadIdx.x == 0) {
+      mbar_arrive_expect_tx(&bar, 2u * (uint32_t)n * row_bytes);
+      for (int i = 0; i < n; ++i) {
+        bulk_g2s(sm + (size_t)i * row_bytes, ht + (t0 + i) * D, row_bytes, &bar);
+        bulk_g2s(sm + (size_t)(tpc + i) * row_bytes, hp + (t0 + i) * D, row_bytes, &bar);
+      }
+    }
+    // every thread waits for the chunk (bounded); a timeout skips the chunk
+    const bool ok = mbar_wait_bounded(&bar, phase, nullptr, status);
+    if (ok) {
+      for (int i = warp; i < n; i += kWarpsPerCta) {
+        const T* a = s_t + (size_t)i * D;
+        const T* p = s_p + (size_t)i * D;
+        float dd = 0.f, pp = 0.f;
+        if (sizeof(T) == 2) {
+          const uint4* a4 = reinterpret_cast<const uint4*>(a);
+          const uint4* p4 = reinterpret_cast<const uint4*>(p);
+          for (int k = lane; k < (int)(row_bytes / 16); k += 32) {
+            const uint4 ra = a4[k], rp = p4[k];
+            const uint32_t wa[4] = {ra.x, ra.y, ra.z, ra.w};
+            const uint32_t wp[4] = {rp.x, rp.y, rp.z, rp.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float d0 = bf16_lo(wa[e]) - bf16_lo(wp[e]), d1 = bf16_hi(wa[e]) - bf16_hi(wp[e]);
+              dd = fmaf(d0, d0, fmaf(d1, d1, dd));
+              pp = fmaf(bf16_lo(wp[e]), bf16_lo(wp[e]), fmaf(bf16_hi(wp[e]), bf16_hi(wp[e]), pp));
+            }
+          }
+        } else {
+          const float4* a4 = reinterpret_cast<const float4*>(a);
+          const float4* p4 = reinterpret_cast<const float4*>(p);
+          for (int k = lane; k < (int)(row_bytes / 16); k += 32) {
+            const float4 ra = a4[k], rp = p4[k];
+            const float av[4] = {ra.x, ra.y, ra.z, ra.w}, pv[4] = {rp.x, rp.y, rp.z, rp.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float d0 = av[e] - pv[e];
+              dd = fmaf(d0, d0, dd);
+              pp = fmaf(pv[e], pv[e], pp);
+            }
+          }
+        }
+        dd = warp_sum(dd);
+        pp = warp_sum(pp);
+        if (lane == 0) V[t0 + i] = sqrtf(dd) / (sqrtf(pp) + eps);
+      }
+    }
+    __syncthreads();   // the buffer is reused by the next chunk
+  }
+}
+
 struct SnapPtrs {
   const void* p[kMaxSnapshots];
 };
@@ -179,11 +271,40 @@ int grid_for(int64_t ntok, int num_sms) {
 
 }  // namespace
 
+template <typename T>
+cudaError_t launch_staged(const void* ht, const void* hp, int64_t ntok, int D, float eps, float* V,
+                          int num_sms, unsigned int* status, cudaStream_t s) {
+  const size_t row = (size_t)D * sizeof(T);
+  const int tpc = (int)std::min<size_t>(kStageTokens, kStageBytesMax / (2 * row));
+  const size_t smem = 2 * (size_t)tpc * row;
+  static int done[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (!(dev >= 0 && dev < 64 && __atomic_load_n(&done[dev], __ATOMIC_ACQUIRE))) {
+    e = cudaFuncSetAttribute(temporal_staged_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kStageBytesMax);
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < 64) __atomic_store_n(&done[dev], 1, __ATOMIC_RELEASE);
+  }
+  const int64_t nchunks = (ntok + tpc - 1) / tpc;
+  const int grid = (int)std::min<int64_t>(nchunks, (int64_t)std::max(num_sms, 1) * 16);
+  temporal_staged_kernel<T><<<grid, kWarpsPerCta * 32, smem, s>>>(
+      static_cast<const T*>(ht), static_cast<const T*>(hp), ntok, D, tpc, eps, V, status);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_temporal(const void* ht, const void* hp, avits_dtype dt, int B, int N, int D,
-                            float eps, float* V, int num_sms, cudaStream_t s) {
+                            float eps, float* V, int num_sms, unsigned int* status, cudaStream_t s) {
   const int64_t ntok = (int64_t)B * N;
   const int grid = grid_for(ntok, num_sms);
   const bool al = ((reinterpret_cast<uintptr_t>(ht) | reinterpret_cast<uintptr_t>(hp)) & 15u) == 0;
+  const size_t row = (size_t)D * (dt == AVITS_BF16 ? 2 : 4);
+  if (al && row % 16 == 0 && 2 * row <= (size_t)kStageBytesMax) {
+    return dt == AVITS_BF16
+               ? launch_staged<__nv_bfloat16>(ht, hp, ntok, D, eps, V, num_sms, status, s)
+               : launch_staged<float>(ht, hp, ntok, D, eps, V, num_sms, status, s);
+  }
   if (dt == AVITS_BF16) {
     if (al && D % 8 == 0) {
       const int chunks = D / 8;

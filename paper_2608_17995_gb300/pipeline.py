@@ -95,10 +95,28 @@ class TransitionBuffers:
         avits_merge_final(self.mixed, self.pos, self.span, self.full_h, self.full_w, self.full,
                           mode=self.mode, workspace=self.merge_ws, stream=stream)
 
-    def run(self, stream=None, merge=True):
-        self.spatial(stream)
-        self.temporal(stream)
-        self.select(stream)
-        self.upsample(stream)
+    def run(self, stream=None, merge=True, concurrent=False):
+        """The transition on `stream`.  With `concurrent`, the temporal score
+        (HBM-bound) runs on a forked side stream while the spatial score
+        (tensor/MUFU-bound) runs on `stream`; both join before selection.
+        The fork/join is recorded into CUDA graphs when captured."""
+        import torch
+        main = stream if stream is not None else torch.cuda.current_stream()
+        if concurrent:
+            if getattr(self, "_side", None) is None:
+                self._side = torch.cuda.Stream(device=main.device)
+                self._fork = torch.cuda.Event()
+                self._join = torch.cuda.Event()
+            self._fork.record(main)
+            self._side.wait_event(self._fork)
+            self.temporal(self._side)
+            self._join.record(self._side)
+            self.spatial(main)
+            main.wait_event(self._join)
+        else:
+            self.spatial(main)
+            self.temporal(main)
+        self.select(main)
+        self.upsample(main)
         if merge:
-            self.merge(stream)
+            self.merge(main)

@@ -141,6 +141,9 @@ def test_spatial_strided_views_and_accumulate(av, orc):
 
 
 def test_spatial_deterministic_and_workspace_clean(av):
+    """Repeated calls on one workspace give bit-identical A.  A is refilled
+    with NaN before every call: a ticket left non-zero by the previous call
+    would keep the last-arriver merge from running and leave NaN behind."""
     import torch
     from paper_2608_17995_gb300 import SpatialWorkspace
     from paper_2608_17995_gb300.workloads import make_transition
@@ -148,16 +151,14 @@ def test_spatial_deterministic_and_workspace_clean(av):
     q, k = _dev(tr.q_img, "bf16"), _dev(tr.k_all, "bf16")
     ws = SpatialWorkspace()
     outs = []
-    for _ in range(3):
-        A = torch.empty(tr.B, tr.M, dtype=torch.float32, device="cuda")
+    for _ in range(4):
+        A = torch.full((tr.B, tr.M), float("nan"), dtype=torch.float32, device="cuda")
         av.avits_score_spatial(q, k, tr.L, tr.softmax_scale, A, workspace=ws)
         outs.append(A.cpu())
-        torch.cuda.synchronize()
-        nbytes = av.avits_score_spatial_workspace(av.BF16, tr.B, tr.H, tr.M, tr.Nk, tr.d)
-        # the ticket counters at the head of the workspace are back to zero
-        assert int(ws.buf[: min(nbytes, 4096)].view(torch.int32)[:96 + 4].abs().sum()) == 0
     assert _status(av) == 0
-    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[1], outs[2])
+    for o in outs:
+        assert not torch.isnan(o).any()
+        assert torch.equal(o, outs[0])
 
 
 # ------------------------------------------------------------ temporal ----
