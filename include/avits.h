@@ -111,6 +111,41 @@ avits_status avits_score_spatial(const void* q_img, const void* k_all, avits_dty
 size_t avits_score_spatial_workspace(avits_dtype dt, int B, int H, int M, int Nk, int d);
 
 /* ------------------------------------------------------------------------
+ * avits_score_spatial without a workspace argument, for callers that may not
+ * allocate device memory where they call this (they only hold their input
+ * and output pointers and a stream, e.g. inside an inference engine's plugin
+ * enqueue or a runtime's custom-op callback, where cudaMalloc would
+ * synchronise the device or is not allowed).  The paper has no counterpart:
+ * this is a deployment convenience of this library.
+ *
+ * Same arguments and results as avits_score_spatial (tensor-core path only:
+ * bf16, d in {64,128}, 16-byte aligned layout; anything else returns
+ * AVITS_ERR_UNSUPPORTED).  The scratch is a fixed array inside the library,
+ * avits_score_spatial_noalloc_limit() bytes (8 MiB) per GPU, held by every
+ * GPU that loads the library until the process exits.  A call whose shapes
+ * need more returns AVITS_ERR_INVALID_ARG before launching anything, with the
+ * sizes in avits_score_spatial_noalloc_error().  The call allocates nothing.
+ *  - The first call on each device looks up the array's device address;
+ *    make that first call before any stream capture on that device.
+ *  - All calls on a device share the one array: calls that may overlap on
+ *    the GPU (other streams, other host threads) race and must be ordered
+ *    by the caller.  Nothing in the array needs clearing between calls.
+ * ---------------------------------------------------------------------- */
+avits_status avits_score_spatial_noalloc(const void* q_img, const void* k_all, avits_dtype dt,
+                                         int B, int H, int M, int Nk, int L, int d,
+                                         int64_t q_sb, int64_t q_sh, int64_t q_sn,
+                                         int64_t k_sb, int64_t k_sh, int64_t k_sn,
+                                         float softmax_scale, float weight, int accumulate,
+                                         float* A, float* lse_opt, void* stream);
+
+/* Bytes of the static scratch array of avits_score_spatial_noalloc. */
+size_t avits_score_spatial_noalloc_limit(void);
+
+/* Why the last avits_score_spatial_noalloc call on this thread was refused
+ * for its size ("" otherwise). */
+const char* avits_score_spatial_noalloc_error(void);
+
+/* ------------------------------------------------------------------------
  * Temporal importance.  Sec. 3.3.2 scores a token by how much its feature
  * moves across the collected denoising steps.  This call takes the two most
  * recent snapshots and returns the relative step change

@@ -257,3 +257,31 @@ def avits_merge_final(mixed, pos, span, full_h: int, full_w: int, out_full, mode
                                  _ptr(workspace), ws_bytes, _stream(stream))
     _check("avits_merge_final", rc)
     return out_full
+
+
+def avits_score_spatial_noalloc(q_img, k_all, L: int, softmax_scale: float, A, weight: float = 1.0,
+                                accumulate: bool = False, lse=None, stream=None):
+    """avits_score_spatial without a workspace: the library's fixed device
+    scratch is used instead (for callers that cannot allocate where they call
+    this, e.g. inside an engine plugin's enqueue).  Same arguments otherwise;
+    bf16 tensor-core shapes only.  Calls on one device must not overlap."""
+    L_ = lib()
+    fn = L_.avits_score_spatial_noalloc
+    if fn.restype is not ctypes.c_int or not fn.argtypes:
+        vp, i32, i64, f32 = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float
+        fn.argtypes = [vp, vp, i32, i32, i32, i32, i32, i32, i32, i64, i64, i64, i64, i64, i64,
+                       f32, f32, i32, vp, vp, vp]
+        fn.restype = ctypes.c_int
+        L_.avits_score_spatial_noalloc_error.restype = ctypes.c_char_p
+        L_.avits_score_spatial_noalloc_limit.restype = ctypes.c_size_t
+    B, H, M, d = q_img.shape
+    Nk = k_all.shape[2]
+    rc = fn(_ptr(q_img), _ptr(k_all), _dtype_code(q_img), B, H, M, Nk, L, d,
+            q_img.stride(0), q_img.stride(1), q_img.stride(2),
+            k_all.stride(0), k_all.stride(1), k_all.stride(2),
+            float(softmax_scale), float(weight), 1 if accumulate else 0,
+            _ptr(A), _ptr(lse), _stream(stream))
+    if rc != 0:
+        raise AvitsError("avits_score_spatial_noalloc", rc,
+                         L_.avits_score_spatial_noalloc_error().decode())
+    return A
