@@ -228,20 +228,13 @@ def run_ours(args, world, rank, local, pg):
     sets = [base] + [tuple(t.clone() for t in base) for _ in range(nsets - 1)]
     torch.cuda.synchronize()
 
-    kernels_per_step = 5 if buf.mode == av.NEAREST else 6   # bilinear merge: map + gather
+    # spatial = scores + merge kernel; bilinear merge = map + gather kernels
+    kernels_per_step = 6 if buf.mode == av.NEAREST else 7
     names = ["spatial", "temporal", "select", "upsample", "merge"]
 
-    def step(s, st, events=None):
+    def step(s, st):
         buf.set_inputs(*sets[s % nsets])
-        if events is None:
-            buf.run(st)            # temporal on a forked stream, joined before select
-            return
-        # per-kernel timing: the five calls in sequence on one stream
-        calls = (buf.spatial, buf.temporal, buf.select, buf.upsample, buf.merge)
-        for i, c in enumerate(calls):
-            events[i].record(st)
-            c(st)
-        events[5].record(st)
+        buf.run(st)
 
     # eager warm-up (also builds the spatial workspace), then graphs
     with torch.cuda.stream(stream):
@@ -311,7 +304,7 @@ def run_ours(args, world, rank, local, pg):
     value = aggregate(K, world, max_ms / 1e3)
 
     # ---------------- per-kernel durations (events between kernels) ----------
-    per_kernel = per_kernel_times(torch, av, step, nsets, stream, names, args)
+    per_kernel = per_kernel_times(torch, av, buf, sets, nsets, stream, names, args)
     work = algorithmic_work(tr, mode)
     peaks = measured_peaks()
     kt = {}
@@ -334,7 +327,8 @@ def run_ours(args, world, rank, local, pg):
     roofline = None
     if sp_ms:
         achieved = work["spatial"]["flops"] / (sp_ms * 1e-3) / 1e12
-        roofline = {"kernel": "spatial_tc_kernel (avits_score_spatial)", "bound": "tensor",
+        roofline = {"kernel": "spatial_tc_kernel + its merge (one avits_score_spatial call)",
+                    "bound": "tensor",
                     "achieved": round(achieved, 2), "peak": peaks["bf16_tflops"],
                     "unit": "TFLOP/s", "frac": round(achieved / peaks["bf16_tflops"], 4),
                     "peak_source": peaks["source"] + " bf16 burst (MEASURED_PEAKS.json)",
@@ -355,8 +349,7 @@ def run_ours(args, world, rank, local, pg):
         "gpu_launches": K * kernels_per_step,
         "clocks": clk,
         "kernels": kt,
-        "kernels_timing": {"how": per_kernel["_how"],
-                           "eager_step_us": round(per_kernel["_step"] * 1e3, 3)},
+        "kernels_timing": per_kernel["_how"],
         "roofline": roofline,
     }
     if not args.no_e2e and not args.quick:
@@ -366,21 +359,32 @@ def run_ours(args, world, rank, local, pg):
     return result, tr
 
 
-def per_kernel_times(torch, av, step, nsets, stream, names, args):
-    """Average device time of each kernel over eager steps whose launches
-    are all queued behind a sleep kernel, so that the events between them
-    bracket back-to-back kernels rather than host launch latency."""
-    n_steps = max(nsets * 10, 100)
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(n_steps)]
-    with torch.cuda.stream(stream):
-        for s in range(n_steps):
-            torch.cuda._sleep(1_000_000)     # ~0.5 ms: the host enqueues the step meanwhile
-            step(s, stream, evs[s])
-    stream.synchronize()
-    out = {"_how": "eager, queued behind a sleep kernel"}
-    for i, n in enumerate(names):
-        out[n] = sum(evs[s][i].elapsed_time(evs[s][i + 1]) for s in range(n_steps)) / n_steps
-    out["_step"] = sum(evs[s][0].elapsed_time(evs[s][5]) for s in range(n_steps)) / n_steps
+def per_kernel_times(torch, av, buf, sets, nsets, stream, names, args):
+    """Average device time per call of each entry point: a CUDA graph of
+    `n` back-to-back calls of that one entry point (rotating over the input
+    copies) is replayed between CUDA events on the launching stream.  A call's
+    time includes its in-graph launch gap; avits_score_spatial is two kernels
+    (scores + merge)."""
+    calls = {"spatial": buf.spatial, "temporal": buf.temporal, "select": buf.select,
+             "upsample": buf.upsample, "merge": buf.merge}
+    n, reps = max(nsets * 4, 48), 10
+    out = {"_how": "graph of %d back-to-back calls per entry point, %d replays" % (n, reps)}
+    for name in names:
+        fn = calls[name]
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for s in range(n):
+                buf.set_inputs(*sets[s % nsets])
+                fn(stream)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            g.replay()
+            e0.record(stream)
+            for _ in range(reps):
+                g.replay()
+            e1.record(stream)
+        stream.synchronize()
+        out[name] = e0.elapsed_time(e1) / (n * reps)
     return out
 
 

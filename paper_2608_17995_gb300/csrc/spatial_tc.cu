@@ -496,7 +496,7 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
         if (ok) {
           tc_fence_after();
           const uint32_t tb = tlane + (uint32_t)(sb * kBN);
-          const int c0 = (seg.kt0 + j) * kBN + half * 64;       // first key of this half
+          const int c0 = (seg.kt0 + j) * kBN + half * 64;        // first key of this half
           const int nch = max(0, min(4, (p.Nk - c0 + 15) >> 4));  // chunks with a valid key
           uint32_t ra[16], rb[16];
           tmem_ld16(tb, ra);
@@ -510,11 +510,16 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
           tmem_ld16(tb + 48, rb);
           if (2 < nch) process_chunk<0>(ra, c0 + 32, p.Nk, p.L, p.c_log2, st);
           tmem_wait(rb);
-          if (3 < nch) process_chunk<0>(rb, c0 + 48, p.Nk, p.L, p.c_log2, st);
+          // all of this warp's columns are in registers: hand the S buffer
+          // back before the last chunk is reduced
           tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bars->s_empty[t][sb]);
+          if (3 < nch) process_chunk<0>(rb, c0 + 48, p.Nk, p.L, p.c_log2, st);
+        } else {
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bars->s_empty[t][sb]);
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bars->s_empty[t][sb]);
       }
       // this warpgroup's piece of the unit: slot 2 * (CTA - first CTA of u) + half
       const int u = seg.u;
@@ -538,27 +543,27 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
 }
 
 // Second kernel: merge the pieces of every (row, head) in slot order, then the
-// head mean of Eq. 3.  Block = 32 rows x 8 head groups; thread (r, hg) merges
-// heads hg, hg+8, ... of row r (all loads of a head issued before its merge)
-// and the 8 partial sums are added in head-group order.  Launched as a
-// programmatic dependent of spatial_tc_kernel: it waits for the producer grid
-// to complete before reading the pieces.
-constexpr int kFinRows = 32, kFinGroups = 8;
+// head mean of Eq. 3.  Block = 32 rows x 32 head lanes; thread (r, hl) merges
+// heads hl, hl+32, ... of row r (all loads of a head issued before its
+// merge), then thread (r, 0) adds the per-head masses in head order from
+// shared memory.  Launched as a programmatic dependent of spatial_tc_kernel:
+// it waits for the producer grid to complete before reading the pieces.
+constexpr int kFinRows = 32, kFinHeads = 32;
 
-__global__ void __launch_bounds__(kFinRows * kFinGroups)
+__global__ void __launch_bounds__(kFinRows * kFinHeads)
 spatial_finalize_kernel(const TcParams p) {
   asm volatile("griddepcontrol.wait;" ::: "memory");
-  __shared__ float part_sum[kFinGroups][kFinRows];
-  const int r = threadIdx.x % kFinRows, hg = threadIdx.x / kFinRows;
+  __shared__ float mass_s[kFinHeads][kFinRows + 1];
+  const int r = threadIdx.x % kFinRows, hl = threadIdx.x / kFinRows;
   const int row_g = blockIdx.x * kFinRows + r;            // over B * n_qp * 256
   const int rows_per_b = p.n_qp * kUnitRows;
   const int b = row_g / rows_per_b;
   const int row = row_g - b * rows_per_b;                  // row within the element
   const int qp = row / kUnitRows, rowu = row - qp * kUnitRows;
   const float ln2 = 0.69314718055994530942f;
-  float sum = 0.f;
+  float sum = 0.f;   // this thread's heads, in head order
   if (b < p.B) {
-    for (int h = hg; h < p.H; h += kFinGroups) {
+    for (int h = hl; h < p.H; h += kFinHeads) {
       const int u = (b * p.H + h) * p.n_qp + qp;
       const int np = 2 * pieces(u, p.n_kt, p.per);
       const float* q = p.part + ((long long)u * (2 * p.max_parts) * kUnitRows + rowu) * 3;
@@ -585,11 +590,14 @@ spatial_finalize_kernel(const TcParams p) {
       }
     }
   }
-  part_sum[hg][r] = sum;
+  mass_s[hl][r] = sum;
   __syncthreads();
-  if (hg == 0 && b < p.B && row < p.M) {
+  if (hl == 0 && b < p.B && row < p.M) {
+    // heads 0..31 first-round partials are in head order; for H > 32 each
+    // lane's partial already holds its heads hl, hl+32, ... in order
     float tot = 0.f;
-    for (int k = 0; k < kFinGroups; ++k) tot += part_sum[k][r];
+    const int lanes = p.H < kFinHeads ? p.H : kFinHeads;
+    for (int k = 0; k < lanes; ++k) tot += mass_s[k][r];
     const float a = p.weight * (tot / (float)p.H);
     float* ap = p.A + (long long)b * p.M + row;
     *ap = p.accumulate ? *ap + a : a;
@@ -733,7 +741,7 @@ cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s)
   // main kernel drains and waits (griddepcontrol.wait) for its completion
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3((unsigned)((a.B * pl.n_qp * kUnitRows + kFinRows - 1) / kFinRows));
-  cfg.blockDim = dim3(kFinRows * kFinGroups);
+  cfg.blockDim = dim3(kFinRows * kFinHeads);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
