@@ -161,6 +161,26 @@ avits_status avits_score_temporal(const void* h_t, const void* h_prev, avits_dty
                                   int B, int N, int D, float eps, float* V, void* stream);
 
 /* ------------------------------------------------------------------------
+ * Both scores of one transition in one call: avits_score_spatial followed by
+ * avits_score_temporal on the same stream, with the same arguments and
+ * results as the two calls (h_t / h_prev are [B,M,D]: the M scored tokens).
+ * On the tensor-core path the temporal kernel is launched as a programmatic
+ * dependent of the spatial kernel and streams the two snapshots from HBM
+ * while the spatial kernel is tensor/MUFU-bound, instead of after it.  Its
+ * inputs must be complete when the call is made (as for any stream-ordered
+ * call); all results are complete for the next call on the stream.
+ * ---------------------------------------------------------------------- */
+avits_status avits_score_spatiotemporal(const void* q_img, const void* k_all, avits_dtype dt,
+                                        int B, int H, int M, int Nk, int L, int d,
+                                        int64_t q_sb, int64_t q_sh, int64_t q_sn,
+                                        int64_t k_sb, int64_t k_sh, int64_t k_sn,
+                                        float softmax_scale, float weight, int accumulate,
+                                        float* A, float* lse_opt,
+                                        void* workspace, size_t ws_bytes,
+                                        const void* h_t, const void* h_prev, int D, float eps,
+                                        float* V, void* stream);
+
+/* ------------------------------------------------------------------------
  * Paper-form temporal importance, Sec. 3.3.2 Eq. 6-7: for each token the
  * unbiased sample variance over N_T snapshots of every channel, averaged
  * over the D channels.

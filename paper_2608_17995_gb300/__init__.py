@@ -26,6 +26,7 @@ from . import _build
 __all__ = [
     "AvitsError", "build", "lib", "library_path",
     "avits_score_spatial", "avits_score_spatial_workspace", "avits_score_temporal",
+    "avits_score_spatiotemporal",
     "avits_score_temporal_var", "avits_fuse_select", "avits_selective_upsample",
     "avits_merge_final", "avits_merge_final_workspace", "avits_device_status",
     "avits_status_string", "avits_version", "SpatialWorkspace",
@@ -70,6 +71,9 @@ def lib():
                                 i64, f32, f32, i32, vp, vp, vp, sz, vp],
         "avits_score_spatial_workspace": [i32, i32, i32, i32, i32, i32],
         "avits_score_temporal": [vp, vp, i32, i32, i32, i32, f32, vp, vp],
+        "avits_score_spatiotemporal": [vp, vp, i32, i32, i32, i32, i32, i32, i32, i64, i64, i64,
+                                       i64, i64, i64, f32, f32, i32, vp, vp, vp, sz, vp, vp, i32,
+                                       f32, vp, vp],
         "avits_score_temporal_var": [vp, i32, i32, i32, i32, i32, vp, vp],
         "avits_fuse_select": [vp, vp, i32, i32, f32, f32, i32, vp, vp, vp, vp, vp],
         "avits_selective_upsample": [vp, i32, i32, i32, i32, i32, i32, i32, vp, vp, vp, vp, i32,
@@ -201,6 +205,36 @@ def avits_score_spatial(q_img, k_all, L: int, softmax_scale: float, A, weight: f
         _ptr(A), _ptr(lse), _ptr(wbuf), wbytes, _stream(stream))
     _check("avits_score_spatial", rc)
     return A
+
+
+def avits_score_spatiotemporal(q_img, k_all, L: int, softmax_scale: float, A, h_t, h_prev, V,
+                               weight: float = 1.0, accumulate: bool = False, lse=None,
+                               eps: float = 1e-6, workspace: Optional[SpatialWorkspace] = None,
+                               stream=None):
+    """avits_score_spatial + avits_score_temporal in one call (the temporal
+    kernel overlaps the spatial one on the tensor-core path)."""
+    B, H, M, d = q_img.shape
+    Nk = k_all.shape[2]
+    D = h_t.shape[2]
+    if q_img.stride(3) != 1 or k_all.stride(3) != 1:
+        raise ValueError("the head-dim axis must be contiguous")
+    if not (h_t.is_contiguous() and h_prev.is_contiguous()) or tuple(h_t.shape[:2]) != (B, M):
+        raise ValueError("h_t / h_prev must be contiguous [B, M, D]")
+    dt = _dtype_code(q_img)
+    need = int(lib().avits_score_spatial_workspace(dt, B, H, M, Nk, d))
+    if workspace is None:
+        key = (q_img.device.index, _stream(stream))
+        workspace = _default_ws.setdefault(key, SpatialWorkspace(q_img.device))
+    wbuf, wbytes = workspace.get(need)
+    rc = lib().avits_score_spatiotemporal(
+        _ptr(q_img), _ptr(k_all), dt, B, H, M, Nk, L, d,
+        q_img.stride(0), q_img.stride(1), q_img.stride(2),
+        k_all.stride(0), k_all.stride(1), k_all.stride(2),
+        float(softmax_scale), float(weight), 1 if accumulate else 0,
+        _ptr(A), _ptr(lse), _ptr(wbuf), wbytes, _ptr(h_t), _ptr(h_prev), D, float(eps), _ptr(V),
+        _stream(stream))
+    _check("avits_score_spatiotemporal", rc)
+    return A, V
 
 
 def avits_score_temporal(h_t, h_prev, V, eps: float = 1e-6, stream=None):

@@ -118,6 +118,41 @@ avits_status avits_score_temporal(const void* h_t, const void* h_prev, avits_dty
                                      status_word(), static_cast<cudaStream_t>(stream)));
 }
 
+avits_status avits_score_spatiotemporal(const void* q_img, const void* k_all, avits_dtype dt,
+                                        int B, int H, int M, int Nk, int L, int d, int64_t q_sb,
+                                        int64_t q_sh, int64_t q_sn, int64_t k_sb, int64_t k_sh,
+                                        int64_t k_sn, float softmax_scale, float weight,
+                                        int accumulate, float* A, float* lse_opt, void* workspace,
+                                        size_t ws_bytes, const void* h_t, const void* h_prev,
+                                        int D, float eps, float* V, void* stream) {
+  if (!q_img || !k_all || !A || !h_t || !h_prev || !V || !valid_dtype(dt))
+    return AVITS_ERR_INVALID_ARG;
+  if (B <= 0 || H <= 0 || M <= 0 || Nk <= 0 || d <= 0 || L < 0 || L > Nk || Nk < M || D <= 0)
+    return AVITS_ERR_INVALID_ARG;
+  if (!(softmax_scale > 0.f) || !(softmax_scale < 3.0e38f) || !(eps >= 0.f))
+    return AVITS_ERR_INVALID_ARG;
+  if (q_sn < d || k_sn < d || q_sh < 0 || k_sh < 0 || q_sb < 0 || k_sb < 0)
+    return AVITS_ERR_INVALID_ARG;
+  SpatialArgs a{q_img, k_all, dt, B, H, M, Nk, L, d, q_sb, q_sh, q_sn, k_sb, k_sh, k_sn,
+                softmax_scale, weight, accumulate ? 1 : 0, A, lse_opt, workspace, ws_bytes,
+                status_word()};
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int sms = num_sms_current();
+  if (spatial_tc_eligible(a)) {
+    if (ws_bytes < spatial_tc_workspace(B, H, M, Nk, d, sms) || !workspace)
+      return AVITS_ERR_INVALID_ARG;
+    unsigned int* st = a.status;
+    const LaunchHook temporal = [=](cudaStream_t ss) {
+      return launch_temporal_overlapped(h_t, h_prev, dt, B, M, D, eps, V, sms, st, ss);
+    };
+    return cuda_status(launch_spatial_tc(a, sms, s, &temporal));
+  }
+  if (d > 256) return AVITS_ERR_UNSUPPORTED;
+  cudaError_t e = launch_spatial_simt(a, s);
+  if (e == cudaSuccess) e = launch_temporal(h_t, h_prev, dt, B, M, D, eps, V, sms, a.status, s);
+  return cuda_status(e);
+}
+
 avits_status avits_score_temporal_var(const void* const* snaps, int n_t, avits_dtype dt, int B,
                                       int N, int D, float* V, void* stream) {
   if (!snaps || !V || !valid_dtype(dt)) return AVITS_ERR_INVALID_ARG;

@@ -3,6 +3,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <functional>
 #include <cuda_runtime.h>
 
 #include "avits.h"
@@ -32,7 +33,10 @@ struct SpatialArgs {
 // layout is not eligible (the caller then uses the CUDA-core path).
 bool spatial_tc_eligible(const SpatialArgs& a);
 size_t spatial_tc_workspace(int B, int H, int M, int Nk, int d, int num_sms);
-cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s);
+// Launches issued between the main spatial kernel and its merge kernel.
+using LaunchHook = std::function<cudaError_t(cudaStream_t)>;
+cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s,
+                              const LaunchHook* between = nullptr);
 
 // CUDA-core path (fp32 or bf16, any d <= 256): one warp per query row.
 cudaError_t launch_spatial_simt(const SpatialArgs& a, cudaStream_t s);
@@ -40,6 +44,11 @@ cudaError_t launch_spatial_simt(const SpatialArgs& a, cudaStream_t s);
 // ---- temporal ---------------------------------------------------------------
 cudaError_t launch_temporal(const void* ht, const void* hp, avits_dtype dt, int B, int N, int D,
                             float eps, float* V, int num_sms, unsigned int* status, cudaStream_t s);
+// The temporal score as a programmatic dependent of the kernel just launched
+// on `s`: one CTA per SM running beside it, waiting for it before exiting.
+cudaError_t launch_temporal_overlapped(const void* ht, const void* hp, avits_dtype dt, int B,
+                                       int N, int D, float eps, float* V, int num_sms,
+                                       unsigned int* status, cudaStream_t s);
 constexpr int kMaxSnapshots = 16;
 cudaError_t launch_temporal_var(const void* const* snaps, int n_t, avits_dtype dt, int B, int N,
                                 int D, float* V, int num_sms, cudaStream_t s);

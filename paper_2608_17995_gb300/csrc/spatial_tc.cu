@@ -683,8 +683,19 @@ cudaError_t set_smem_once() {
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev >= 0 && dev < 64 && __atomic_load_n(&done[dev], __ATOMIC_ACQUIRE)) return cudaSuccess;
-  e = cudaFuncSetAttribute(spatial_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           smem_bytes<128>());
+  // one carveout (all shared) for every kernel of the path, so that kernels
+  // launched as programmatic dependents can share an SM with this one
+  e = cudaFuncSetAttribute(spatial_tc_kernel<128>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(spatial_tc_kernel<64>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(spatial_finalize_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(spatial_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             smem_bytes<128>());
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(spatial_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              smem_bytes<64>());
@@ -711,7 +722,8 @@ size_t spatial_tc_workspace(int B, int H, int M, int Nk, int d, int num_sms) {
   return make_plan(B, H, M, Nk, num_sms).bytes;
 }
 
-cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s) {
+cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s,
+                              const LaunchHook* between) {
   const Plan pl = make_plan(a.B, a.H, a.M, a.Nk, num_sms);
   if (a.ws_bytes < pl.bytes || a.ws == nullptr) return cudaErrorInvalidValue;
   CUtensorMap mq, mk;
@@ -737,6 +749,12 @@ cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s)
     spatial_tc_kernel<64><<<pl.grid, kThreads, smem_bytes<64>(), s>>>(mq, mk, p);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  if (between) {
+    // work that may overlap the main kernel (launched as its programmatic
+    // dependent); it must not complete before the main kernel does
+    e = (*between)(s);
+    if (e != cudaSuccess) return e;
+  }
   // the merge runs as a programmatic dependent: it may be scheduled while the
   // main kernel drains and waits (griddepcontrol.wait) for its completion
   cudaLaunchConfig_t cfg{};

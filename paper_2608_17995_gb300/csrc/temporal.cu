@@ -149,10 +149,15 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       : "memory");
 }
 
-template <typename T>
+// kOverlapped: launched as a programmatic dependent of a running kernel (the
+// spatial score); lets its own dependents be scheduled, and waits for the
+// running kernel to finish before exiting so that a dependent of this grid
+// also sees that kernel's results.
+template <typename T, bool kOverlapped>
 __global__ void __launch_bounds__(kWarpsPerCta * 32)
 temporal_staged_kernel(const T* __restrict__ ht, const T* __restrict__ hp, int64_t ntok, int D,
                        int tpc, float eps, float* __restrict__ V, unsigned int* status) {
+  if (kOverlapped && threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   extern __shared__ __align__(128) uint8_t sm[];
   __shared__ __align__(8) uint64_t bar;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -219,6 +224,7 @@ temporal_staged_kernel(const T* __restrict__ ht, const T* __restrict__ hp, int64
     }
     __syncthreads();   // the buffer is reused by the next chunk
   }
+  if (kOverlapped) asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
 struct SnapPtrs {
@@ -271,7 +277,7 @@ int grid_for(int64_t ntok, int num_sms) {
 
 }  // namespace
 
-template <typename T>
+template <typename T, bool kOverlapped = false>
 cudaError_t launch_staged(const void* ht, const void* hp, int64_t ntok, int D, float eps, float* V,
                           int num_sms, unsigned int* status, cudaStream_t s) {
   const size_t row = (size_t)D * sizeof(T);
@@ -282,15 +288,40 @@ cudaError_t launch_staged(const void* ht, const void* hp, int64_t ntok, int D, f
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (!(dev >= 0 && dev < 64 && __atomic_load_n(&done[dev], __ATOMIC_ACQUIRE))) {
-    e = cudaFuncSetAttribute(temporal_staged_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             kStageBytesMax);
+    e = cudaFuncSetAttribute(temporal_staged_kernel<T, false>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, kStageBytesMax);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(temporal_staged_kernel<T, true>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, kStageBytesMax);
+    if (e != cudaSuccess) return e;
+    // the same (all shared) carveout as the spatial kernel it runs beside
+    e = cudaFuncSetAttribute(temporal_staged_kernel<T, true>,
+                             cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared);
     if (e != cudaSuccess) return e;
     if (dev >= 0 && dev < 64) __atomic_store_n(&done[dev], 1, __ATOMIC_RELEASE);
   }
   const int64_t nchunks = (ntok + tpc - 1) / tpc;
-  const int grid = (int)std::min<int64_t>(nchunks, (int64_t)std::max(num_sms, 1) * 16);
-  temporal_staged_kernel<T><<<grid, kWarpsPerCta * 32, smem, s>>>(
-      static_cast<const T*>(ht), static_cast<const T*>(hp), ntok, D, tpc, eps, V, status);
+  if (!kOverlapped) {
+    const int grid = (int)std::min<int64_t>(nchunks, (int64_t)std::max(num_sms, 1) * 16);
+    temporal_staged_kernel<T, false><<<grid, kWarpsPerCta * 32, smem, s>>>(
+        static_cast<const T*>(ht), static_cast<const T*>(hp), ntok, D, tpc, eps, V, status);
+    return cudaGetLastError();
+  }
+  // one CTA per SM (it shares the SM with the running kernel's CTA)
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((unsigned)std::min<int64_t>(nchunks, (int64_t)std::max(num_sms, 1)));
+  cfg.blockDim = dim3(kWarpsPerCta * 32);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, temporal_staged_kernel<T, true>, static_cast<const T*>(ht),
+                         static_cast<const T*>(hp), ntok, D, tpc, eps, V, status);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
@@ -334,6 +365,19 @@ cudaError_t launch_temporal(const void* ht, const void* hp, avits_dtype dt, int 
     }
   }
   return cudaGetLastError();
+}
+
+cudaError_t launch_temporal_overlapped(const void* ht, const void* hp, avits_dtype dt, int B,
+                                       int N, int D, float eps, float* V, int num_sms,
+                                       unsigned int* status, cudaStream_t s) {
+  const int64_t ntok = (int64_t)B * N;
+  const bool al = ((reinterpret_cast<uintptr_t>(ht) | reinterpret_cast<uintptr_t>(hp)) & 15u) == 0;
+  const size_t row = (size_t)D * (dt == AVITS_BF16 ? 2 : 4);
+  if (!(al && row % 16 == 0 && 2 * row <= (size_t)kStageBytesMax))
+    return launch_temporal(ht, hp, dt, B, N, D, eps, V, num_sms, status, s);   // stream order
+  return dt == AVITS_BF16
+             ? launch_staged<__nv_bfloat16, true>(ht, hp, ntok, D, eps, V, num_sms, status, s)
+             : launch_staged<float, true>(ht, hp, ntok, D, eps, V, num_sms, status, s);
 }
 
 cudaError_t launch_temporal_var(const void* const* snaps, int n_t, avits_dtype dt, int B, int N,

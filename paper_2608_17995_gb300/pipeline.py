@@ -1,16 +1,17 @@
 """One resolution transition on the device: buffers plus the calls in order.
 
 Plumbing only: it owns the output tensors and the workspaces and issues
-avits_score_spatial -> avits_score_temporal -> avits_fuse_select ->
-avits_selective_upsample -> avits_merge_final on one stream.
+avits_score_spatiotemporal (or avits_score_spatial + avits_score_temporal) ->
+avits_fuse_select -> avits_selective_upsample -> avits_merge_final on one
+stream.
 """
 from __future__ import annotations
 
 import numpy as np
 
 from . import (BILINEAR, NEAREST, SpatialWorkspace, avits_fuse_select, avits_merge_final,
-               avits_merge_final_workspace, avits_score_spatial, avits_score_temporal,
-               avits_selective_upsample)
+               avits_merge_final_workspace, avits_score_spatial, avits_score_spatiotemporal,
+               avits_score_temporal, avits_selective_upsample)
 
 
 def to_device(arr: np.ndarray, dtype: str, device="cuda"):
@@ -78,6 +79,12 @@ class TransitionBuffers:
         avits_score_spatial(self.q, self.k, self.tr.L, self.tr.softmax_scale, self.A,
                             workspace=self.ws, stream=stream)
 
+    def scores(self, stream=None):
+        """Both scores in one call (temporal overlapped with spatial)."""
+        avits_score_spatiotemporal(self.q, self.k, self.tr.L, self.tr.softmax_scale, self.A,
+                                   self.h_t, self.h_prev, self.V, workspace=self.ws,
+                                   stream=stream)
+
     def temporal(self, stream=None):
         avits_score_temporal(self.h_t, self.h_prev, self.V, stream=stream)
 
@@ -95,24 +102,14 @@ class TransitionBuffers:
         avits_merge_final(self.mixed, self.pos, self.span, self.full_h, self.full_w, self.full,
                           mode=self.mode, workspace=self.merge_ws, stream=stream)
 
-    def run(self, stream=None, merge=True, concurrent=False):
-        """The transition on `stream`.  With `concurrent`, the temporal score
-        (HBM-bound) runs on a forked side stream while the spatial score
-        (tensor/MUFU-bound) runs on `stream`; both join before selection.
-        The fork/join is recorded into CUDA graphs when captured."""
+    def run(self, stream=None, merge=True, fused_scores=True):
+        """The transition on one stream: both scores (one call, the temporal
+        kernel overlapping the spatial one, unless fused_scores=False), then
+        selection, selective upsampling and the final merge."""
         import torch
         main = stream if stream is not None else torch.cuda.current_stream()
-        if concurrent:
-            if getattr(self, "_side", None) is None:
-                self._side = torch.cuda.Stream(device=main.device)
-                self._fork = torch.cuda.Event()
-                self._join = torch.cuda.Event()
-            self._fork.record(main)
-            self._side.wait_event(self._fork)
-            self.temporal(self._side)
-            self._join.record(self._side)
-            self.spatial(main)
-            main.wait_event(self._join)
+        if fused_scores:
+            self.scores(main)
         else:
             self.spatial(main)
             self.temporal(main)

@@ -161,6 +161,32 @@ def test_spatial_deterministic_and_workspace_clean(av):
         assert torch.equal(o, outs[0])
 
 
+@pytest.mark.parametrize("name", ["flux1024", "tiny", "batched"])
+def test_spatiotemporal_matches_separate_calls(av, orc, name):
+    """One call for both scores (temporal overlapped with spatial on the
+    tensor-core path) gives the separate calls' results, and the oracle's."""
+    import torch
+    from paper_2608_17995_gb300.workloads import make_transition
+    tr = make_transition(name)
+    q, k = _dev(tr.q_img, tr.dtype), _dev(tr.k_all, tr.dtype)
+    ht, hp = _dev(tr.h_t, tr.dtype), _dev(tr.h_prev, tr.dtype)
+    for _ in range(2):
+        A = torch.full((tr.B, tr.M), float("nan"), device="cuda")
+        V = torch.full((tr.B, tr.M), float("nan"), device="cuda")
+        av.avits_score_spatiotemporal(q, k, tr.L, tr.softmax_scale, A, ht, hp, V)
+        A2 = torch.empty_like(A)
+        V2 = torch.empty_like(V)
+        av.avits_score_spatial(q, k, tr.L, tr.softmax_scale, A2)
+        av.avits_score_temporal(ht, hp, V2)
+        assert _status(av) == 0
+        assert torch.equal(A, A2) and torch.equal(V, V2)
+    rtol = F32_TOL if tr.dtype == "f32" else BF16_RTOL
+    np.testing.assert_allclose(_np(V), orc.score_temporal(tr.h_t, tr.h_prev), rtol=rtol, atol=1e-7)
+    rows = _sample_rows(tr.B, tr.M, 48, seed=3)
+    A_o, _, _ = orc.score_spatial(tr.q_img, tr.k_all, tr.L, tr.softmax_scale, rows=rows)
+    np.testing.assert_allclose(_np(A).ravel()[rows], A_o.ravel()[rows], rtol=rtol, atol=1e-6)
+
+
 # ------------------------------------------------------------ temporal ----
 
 @pytest.mark.parametrize("name", ["tiny", "flux1024", "edit"])
