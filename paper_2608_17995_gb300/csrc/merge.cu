@@ -42,6 +42,7 @@ merge_nearest_kernel(const T* __restrict__ mixed, int B, int N, const int32_t* _
                      const int32_t* __restrict__ span, int fh, int fw, int C, T* __restrict__ out,
                      unsigned int* status) {
   using PV = typename Pix4<T>::V;
+  pdl_wait_then_trigger();
   const int lane = threadIdx.x & 31;
   const int64_t gwarp = (int64_t)blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
   if (gwarp >= (int64_t)B * N) return;
@@ -163,8 +164,12 @@ cudaError_t launch_t(const void* mixed, int B, int N, const int32_t* pos, const 
   if (mode == AVITS_UP_NEAREST) {
     const int64_t warps = (int64_t)B * N;
     const int grid = (int)((warps + kWarpsPerCta - 1) / kWarpsPerCta);
-    merge_nearest_kernel<T><<<grid, kWarpsPerCta * 32, 0, s>>>(
-        static_cast<const T*>(mixed), B, N, pos, span, fh, fw, C, static_cast<T*>(out), status);
+    cudaError_t e = prefer_max_shared<merge_nearest_kernel<T>>();
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(merge_nearest_kernel<T>, dim3(grid), dim3(kWarpsPerCta * 32), 0, s,
+                               static_cast<const T*>(mixed), B, N, pos, span, fh, fw, C,
+                               static_cast<T*>(out), status);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
   }
   int32_t* map = static_cast<int32_t*>(ws);

@@ -70,6 +70,7 @@ fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V, int
   __shared__ uint32_t scan_tot[kWarps];
   __shared__ int sh_nan;
 
+  pdl_wait_then_trigger();
   const int b = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   const float* a = A + (int64_t)b * M;
@@ -284,21 +285,20 @@ cudaError_t launch_fuse_select(const float* A, const float* V, int B, int M, flo
     }
   }
   const int per = (M + kThreads - 1) / kThreads;
-  if (per <= 1)
-    fuse_select_kernel<1><<<B, kThreads, smem, s>>>(A, V, M, alpha, eps, k, S, sel_idx, mask,
-                                                    tok_offset, status);
-  else if (per <= 2)
-    fuse_select_kernel<2><<<B, kThreads, smem, s>>>(A, V, M, alpha, eps, k, S, sel_idx, mask,
-                                                    tok_offset, status);
-  else if (per <= 4)
-    fuse_select_kernel<4><<<B, kThreads, smem, s>>>(A, V, M, alpha, eps, k, S, sel_idx, mask,
-                                                    tok_offset, status);
-  else if (per <= kMaxRegKeys)
-    fuse_select_kernel<kMaxRegKeys><<<B, kThreads, smem, s>>>(A, V, M, alpha, eps, k, S, sel_idx,
-                                                              mask, tok_offset, status);
-  else
-    fuse_select_kernel<0><<<B, kThreads, smem, s>>>(A, V, M, alpha, eps, k, S, sel_idx, mask,
-                                                    tok_offset, status);
+  cudaError_t ce = prefer_max_shared<fuse_select_kernel<1>>();
+  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<2>>();
+  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<4>>();
+  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<kMaxRegKeys>>();
+  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<0>>();
+  if (ce != cudaSuccess) return ce;
+  auto kern = per <= 1   ? fuse_select_kernel<1>
+              : per <= 2 ? fuse_select_kernel<2>
+              : per <= 4 ? fuse_select_kernel<4>
+              : per <= kMaxRegKeys ? fuse_select_kernel<kMaxRegKeys>
+                                   : fuse_select_kernel<0>;
+  cudaError_t e = launch_pdl(kern, dim3(B), dim3(kThreads), smem, s, A, V, M, alpha, eps, k, S,
+                             sel_idx, mask, tok_offset, status);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -338,6 +338,8 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
   const int it_begin = (int)blockIdx.x * p.per;
   const int it_end = min(it_begin + p.per, p.total);
   if (it_begin >= it_end) return;   // block-uniform
+  // Q and K may come from the kernel before this one on the stream
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 
   if (threadIdx.x == 0) {
     for (int t = 0; t < kQTiles; ++t) mbar_init(&bars->q_full[t], 1);
@@ -744,9 +746,12 @@ cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s,
   cudaError_t e = set_smem_once();
   if (e != cudaSuccess) return e;
   if (a.d == 128)
-    spatial_tc_kernel<128><<<pl.grid, kThreads, smem_bytes<128>(), s>>>(mq, mk, p);
+    e = launch_pdl(spatial_tc_kernel<128>, dim3(pl.grid), dim3(kThreads), smem_bytes<128>(), s, mq,
+                   mk, p);
   else
-    spatial_tc_kernel<64><<<pl.grid, kThreads, smem_bytes<64>(), s>>>(mq, mk, p);
+    e = launch_pdl(spatial_tc_kernel<64>, dim3(pl.grid), dim3(kThreads), smem_bytes<64>(), s, mq,
+                   mk, p);
+  if (e != cudaSuccess) return e;
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if (between) {

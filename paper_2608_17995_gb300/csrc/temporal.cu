@@ -157,7 +157,13 @@ template <typename T, bool kOverlapped>
 __global__ void __launch_bounds__(kWarpsPerCta * 32)
 temporal_staged_kernel(const T* __restrict__ ht, const T* __restrict__ hp, int64_t ntok, int D,
                        int tpc, float eps, float* __restrict__ V, unsigned int* status) {
-  if (kOverlapped && threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  if (kOverlapped) {
+    // beside a running kernel: its inputs were complete before that kernel
+    // started; let the dependents of this grid be scheduled
+    if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  } else {
+    pdl_wait_then_trigger();
+  }
   extern __shared__ __align__(128) uint8_t sm[];
   __shared__ __align__(8) uint64_t bar;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -302,10 +308,14 @@ cudaError_t launch_staged(const void* ht, const void* hp, int64_t ntok, int D, f
     if (dev >= 0 && dev < 64) __atomic_store_n(&done[dev], 1, __ATOMIC_RELEASE);
   }
   const int64_t nchunks = (ntok + tpc - 1) / tpc;
+  e = prefer_max_shared<temporal_staged_kernel<T, false>>();
+  if (e != cudaSuccess) return e;
   if (!kOverlapped) {
     const int grid = (int)std::min<int64_t>(nchunks, (int64_t)std::max(num_sms, 1) * 16);
-    temporal_staged_kernel<T, false><<<grid, kWarpsPerCta * 32, smem, s>>>(
-        static_cast<const T*>(ht), static_cast<const T*>(hp), ntok, D, tpc, eps, V, status);
+    e = launch_pdl(temporal_staged_kernel<T, false>, dim3(grid), dim3(kWarpsPerCta * 32), smem, s,
+                   static_cast<const T*>(ht), static_cast<const T*>(hp), ntok, D, tpc, eps, V,
+                   status);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
   }
   // one CTA per SM (it shares the SM with the running kernel's CTA)

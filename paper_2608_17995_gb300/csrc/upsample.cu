@@ -65,6 +65,7 @@ upsample_kernel(const T* __restrict__ latent, int B, int M, int gh, int gw, int 
                 int32_t* __restrict__ out_span, int32_t* __restrict__ out_src_tok,
                 int8_t* __restrict__ out_src_sub) {
   using PV = typename Pix4<T>::V;
+  pdl_wait_then_trigger();
   const int lane = threadIdx.x & 31;
   const int64_t gwarp = (int64_t)blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
   if (gwarp >= (int64_t)B * M) return;
@@ -146,14 +147,15 @@ cudaError_t launch_t(const void* latent, int B, int M, int gh, int gw, int C,
   const int64_t warps = (int64_t)B * M;
   const int grid = (int)((warps + kWarpsPerCta - 1) / kWarpsPerCta);
   const int n_out = M + 3 * k;
-  if (mode == AVITS_UP_BILINEAR)
-    upsample_kernel<T, true><<<grid, kWarpsPerCta * 32, 0, s>>>(
-        static_cast<const T*>(latent), B, M, gh, gw, C, pos_in, span_in, mask, tok_offset, n_out,
-        static_cast<T*>(out), out_pos, out_span, out_src_tok, out_src_sub);
-  else
-    upsample_kernel<T, false><<<grid, kWarpsPerCta * 32, 0, s>>>(
-        static_cast<const T*>(latent), B, M, gh, gw, C, pos_in, span_in, mask, tok_offset, n_out,
-        static_cast<T*>(out), out_pos, out_span, out_src_tok, out_src_sub);
+  cudaError_t e = prefer_max_shared<upsample_kernel<T, true>>();
+  if (e == cudaSuccess) e = prefer_max_shared<upsample_kernel<T, false>>();
+  if (e != cudaSuccess) return e;
+  auto kern = (mode == AVITS_UP_BILINEAR) ? upsample_kernel<T, true> : upsample_kernel<T, false>;
+  e = launch_pdl(kern, dim3(grid), dim3(kWarpsPerCta * 32), 0, s,
+                             static_cast<const T*>(latent), B, M, gh, gw, C, pos_in, span_in, mask,
+                             tok_offset, n_out, static_cast<T*>(out), out_pos, out_span,
+                             out_src_tok, out_src_sub);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
