@@ -19,14 +19,16 @@
 // of the first) merges the pieces of each (row, head) in slot order and sums
 // the heads in head order, so the result does not depend on CTA timing.
 //
-// Roles (18 warps):
+// Roles (19 warps):
 //   warp 0        TMA producer: Q tile 0, the first K tile, Q tile 1, then the
 //                 K tiles through a 4-stage ring (128-byte swizzle, no
 //                 multicast); each Q tile has its own barrier so the first MMA
 //                 starts after 64 KB rather than 96 KB.
-//   warp 1        MMA issuer: S = Q K^T with tcgen05.mma kind::f16 (bf16 in,
-//                 fp32 accumulate in tensor memory), 128x128 per tile, two S
-//                 buffers per Q tile (all 512 TMEM columns).
+//   warps 1, 18   MMA issuers, one per query tile: S = Q K^T with
+//                 tcgen05.mma kind::f16 (bf16 in, fp32 accumulate in tensor
+//                 memory), 128x128 per tile, two S buffers per Q tile (all 512
+//                 TMEM columns).  A barrier wait in the issuing thread costs
+//                 the tensor pipe a bubble; a second issuer fills it.
 //   warps 2-17    four softmax warpgroups: query tile t and column half c
 //                 (64 of the 128 keys of a tile) per warpgroup, so all 16
 //                 warps work on the same item while the MMA fills the other S
@@ -55,7 +57,8 @@ constexpr int kBN = 128;       // keys per tile
 constexpr int kQTiles = 2;     // query tiles per unit
 constexpr int kUnitRows = kBM * kQTiles;
 constexpr int kSoftmaxWarps = 16;
-constexpr int kThreads = 64 + kSoftmaxWarps * 32;
+constexpr int kMmaWarp1 = 2 + kSoftmaxWarps;            // issuer of query tile 1
+constexpr int kThreads = 96 + kSoftmaxWarps * 32;
 constexpr int kTmemCols = 512;
 constexpr uint32_t kIdesc = (1u << 4)                       // D: fp32
                             | (1u << 7) | (1u << 10)        // A, B: bf16
@@ -75,7 +78,7 @@ struct Bars {
   uint64_t q_full[kQTiles], q_empty;
   uint64_t k_full[8], k_empty[8];
   uint64_t s_full[kQTiles][2], s_empty[kQTiles][2];
-  uint64_t drain;
+  uint64_t drain[kQTiles];
   uint32_t tmem_base;
   int abort;
 };
@@ -246,6 +249,45 @@ __device__ __forceinline__ void exp2_fma2(float x0, float x1, float& e0, float& 
   e1 = __int_as_float(__float_as_int(p1) + (__float_as_int(y1) << 23));
 }
 
+// One chunk of 16 keys that are all valid and all text (kText) or all image
+// keys: the common case, kept free of the masking and boundary logic (a
+// per-chunk branch on the key kind measured ~15% slower on the whole item).
+template <bool kText>
+__device__ __forceinline__ void process_chunk_full(const uint32_t (&r)[16], float c, RowStat& st) {
+  float v[16];
+#pragma unroll
+  for (int e = 0; e < 16; ++e) v[e] = __uint_as_float(r[e]);
+  const float nm = -st.m;
+  float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+  for (int e = 0; e < 16; e += 4) {
+    float x0, x1, x2, x3;
+    ffma2(v[e], v[e + 1], c, nm, x0, x1);
+    ffma2(v[e + 2], v[e + 3], c, nm, x2, x3);
+    fadd2(s0, s1, ex2(x0), ex2(x1));
+    fadd2(s2, s3, ex2(x2), ex2(x3));
+  }
+  fadd2(s0, s1, s2, s3);
+  float cs = s0 + s1;
+  if (!(cs < 0x1p64f)) {
+    // first chunk of a row, a logit 64 log2-units above the running maximum,
+    // or a NaN: take the exact chunk maximum and rescale the running sums
+    float cm = v[0];
+#pragma unroll
+    for (int e = 1; e < 16; ++e) cm = fmaxf(cm, v[e]);
+    const float mx = fmaxf(st.m, cm * c);
+    const float corr = ex2(st.m - mx);
+    st.la *= corr;
+    st.lt *= corr;
+    st.m = mx;
+    cs = 0.f;
+#pragma unroll
+    for (int e = 0; e < 16; ++e) cs += ex2(fmaf(v[e], c, -mx));
+  }
+  st.la += cs;
+  if (kText) st.lt += cs;
+}
+
 // One 16-column chunk whose first key is col0 (< Nk); the last E of its
 // exponentials (E = 0, 2 or 4) are evaluated on the FMA pipe.
 template <int E>
@@ -304,6 +346,42 @@ __device__ __forceinline__ void process_chunk(const uint32_t (&r)[16], int col0,
   }
 }
 
+// Kinds of the 64 keys a softmax warp reduces per item.
+enum ItemKind { kItemImage = 0, kItemText = 1, kItemGeneral = 2 };
+
+// The 64 columns [c0, c0 + 64) of one S buffer for this warp's 32 rows: four
+// 16-column tcgen05.ld, each overlapped with the reduction of the previous
+// chunk.  The S buffer is handed back (arrive on s_empty) as soon as all 64
+// columns are in registers, before the last chunk is reduced.
+template <int kKind>
+__device__ __forceinline__ void softmax_item(uint32_t tb, int c0, int Nk, int L, float c,
+                                             RowStat& st, uint64_t* s_empty, int lane) {
+  uint32_t ra[16], rb[16];
+  const int nch = (kKind == kItemGeneral) ? max(0, min(4, (Nk - c0 + 15) >> 4)) : 4;
+  auto chunk = [&](const uint32_t(&r)[16], int k) {
+    if (kKind == kItemGeneral) {
+      if (k < nch) process_chunk<0>(r, c0 + 16 * k, Nk, L, c, st);
+    } else {
+      process_chunk_full<kKind == kItemText>(r, c, st);
+    }
+  };
+  tmem_ld16(tb, ra);
+  tmem_wait(ra);
+  tmem_ld16(tb + 16, rb);
+  chunk(ra, 0);
+  tmem_wait(rb);
+  tmem_ld16(tb + 32, ra);
+  chunk(rb, 1);
+  tmem_wait(ra);
+  tmem_ld16(tb + 48, rb);
+  chunk(ra, 2);
+  tmem_wait(rb);
+  tc_fence_before();
+  __syncwarp();
+  if (lane == 0) mbar_arrive(s_empty);
+  chunk(rb, 3);
+}
+
 struct Segment {
   int u, kt0, nk;
 };
@@ -343,17 +421,17 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
 
   if (threadIdx.x == 0) {
     for (int t = 0; t < kQTiles; ++t) mbar_init(&bars->q_full[t], 1);
-    mbar_init(&bars->q_empty, 1);
+    mbar_init(&bars->q_empty, kQTiles);   // one commit per MMA issuer
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&bars->k_full[s], 1);
-      mbar_init(&bars->k_empty[s], 1);
+      mbar_init(&bars->k_empty[s], kQTiles);
     }
     for (int t = 0; t < kQTiles; ++t)
       for (int b = 0; b < 2; ++b) {
         mbar_init(&bars->s_full[t][b], 1);
         mbar_init(&bars->s_empty[t][b], 8);   // 8 softmax warps read each tile
       }
-    mbar_init(&bars->drain, 1);
+    for (int t = 0; t < kQTiles; ++t) mbar_init(&bars->drain[t], 1);
     bars->abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -431,12 +509,18 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
         }
       }
     }
-  } else if (warp == 1) {
-    // --------------------------------------------------------- MMA issuer --
+  } else if (warp == 1 || warp == kMmaWarp1) {
+    // -------------------------------------------------------- MMA issuers --
+    // One issuing thread per query tile.  A barrier wait in an issuing thread
+    // stalls that thread's queue of MMAs until the tensor pipe has taken it;
+    // with two issuers the other queue keeps the pipe busy meanwhile.
+    const int t = (warp == 1) ? 0 : 1;
     if (lane == 0) {
       bool ok = true;
       int li = 0;
       int sg = 0;
+      const uint8_t* qa = sQ + t * C::kTileBytes;
+      const uint32_t d_base = tmem + (uint32_t)(t * 2 * kBN);
       for (int it = it_begin; it < it_end && ok;) {
         const Segment seg = segment_at(it, it_end, p.n_kt);
         for (int j = 0; j < seg.nk && ok; ++j, ++li) {
@@ -446,26 +530,21 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
           const uint32_t sph = (uint32_t)((li >> 1) & 1);
           ok = mbar_wait_bounded(&bars->k_full[stage], ph, abort_flag, p.status);
           if (!ok) break;
-          tc_fence_after();
-          for (int t = 0; t < kQTiles; ++t) {
-            if (j == 0) {
-              ok = mbar_wait_bounded(&bars->q_full[t], (uint32_t)(sg & 1), abort_flag, p.status);
-              if (!ok) break;
-            }
-            ok = mbar_wait_bounded(&bars->s_empty[t][sb], sph ^ 1u, abort_flag, p.status);
+          if (j == 0) {
+            ok = mbar_wait_bounded(&bars->q_full[t], (uint32_t)(sg & 1), abort_flag, p.status);
             if (!ok) break;
-            tc_fence_after();
-            const uint32_t d_tmem = tmem + (uint32_t)((t * 2 + sb) * kBN);
-            const uint8_t* qa = sQ + t * C::kTileBytes;
-            const uint8_t* kb = sK + stage * C::kTileBytes;
-#pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const int off = (kk >> 2) * (kBM * 128) + (kk & 3) * 32;
-              mma_bf16(d_tmem, sw128_desc(qa + off), sw128_desc(kb + off), kk > 0 ? 1u : 0u);
-            }
-            mma_commit(&bars->s_full[t][sb]);
           }
+          ok = mbar_wait_bounded(&bars->s_empty[t][sb], sph ^ 1u, abort_flag, p.status);
           if (!ok) break;
+          tc_fence_after();
+          const uint32_t d_tmem = d_base + (uint32_t)(sb * kBN);
+          const uint8_t* kb = sK + stage * C::kTileBytes;
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const int off = (kk >> 2) * (kBM * 128) + (kk & 3) * 32;
+            mma_bf16(d_tmem, sw128_desc(qa + off), sw128_desc(kb + off), kk > 0 ? 1u : 0u);
+          }
+          mma_commit(&bars->s_full[t][sb]);
           mma_commit(&bars->k_empty[stage]);
         }
         if (!ok) break;
@@ -474,8 +553,8 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
         ++sg;
       }
       // all issued MMAs complete before tensor memory is released
-      mma_commit(&bars->drain);
-      mbar_wait_bounded(&bars->drain, 0, nullptr, p.status);
+      mma_commit(&bars->drain[t]);
+      mbar_wait_bounded(&bars->drain[t], 0, nullptr, p.status);
     }
   } else {
     // ---------------------------------------------------- softmax-reduce --
@@ -498,26 +577,15 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
         if (ok) {
           tc_fence_after();
           const uint32_t tb = tlane + (uint32_t)(sb * kBN);
-          const int c0 = (seg.kt0 + j) * kBN + half * 64;        // first key of this half
-          const int nch = max(0, min(4, (p.Nk - c0 + 15) >> 4));  // chunks with a valid key
-          uint32_t ra[16], rb[16];
-          tmem_ld16(tb, ra);
-          tmem_wait(ra);
-          tmem_ld16(tb + 16, rb);
-          if (0 < nch) process_chunk<0>(ra, c0, p.Nk, p.L, p.c_log2, st);
-          tmem_wait(rb);
-          tmem_ld16(tb + 32, ra);
-          if (1 < nch) process_chunk<0>(rb, c0 + 16, p.Nk, p.L, p.c_log2, st);
-          tmem_wait(ra);
-          tmem_ld16(tb + 48, rb);
-          if (2 < nch) process_chunk<0>(ra, c0 + 32, p.Nk, p.L, p.c_log2, st);
-          tmem_wait(rb);
-          // all of this warp's columns are in registers: hand the S buffer
-          // back before the last chunk is reduced
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&bars->s_empty[t][sb]);
-          if (3 < nch) process_chunk<0>(rb, c0 + 48, p.Nk, p.L, p.c_log2, st);
+          const int c0 = (seg.kt0 + j) * kBN + half * 64;   // first key of this half
+          uint64_t* empty = &bars->s_empty[t][sb];
+          // the kind is uniform over the warp: one branch per item
+          if (c0 + 64 <= p.Nk && c0 + 64 <= p.L)
+            softmax_item<kItemText>(tb, c0, p.Nk, p.L, p.c_log2, st, empty, lane);
+          else if (c0 + 64 <= p.Nk && c0 >= p.L)
+            softmax_item<kItemImage>(tb, c0, p.Nk, p.L, p.c_log2, st, empty, lane);
+          else
+            softmax_item<kItemGeneral>(tb, c0, p.Nk, p.L, p.c_log2, st, empty, lane);
         } else {
           __syncwarp();
           if (lane == 0) mbar_arrive(&bars->s_empty[t][sb]);
