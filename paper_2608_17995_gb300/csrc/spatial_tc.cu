@@ -416,10 +416,14 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
   const int it_begin = (int)blockIdx.x * p.per;
   const int it_end = min(it_begin + p.per, p.total);
   if (it_begin >= it_end) return;   // block-uniform
-  // Q and K may come from the kernel before this one on the stream
-  asm volatile("griddepcontrol.wait;" ::: "memory");
 
+  // Prologue that touches no global data: it overlaps the tail of the kernel
+  // before this one on the stream (programmatic dependent launch).  The
+  // tensor maps are kernel parameters; fetching them early takes their
+  // latency off the first TMA copy.
   if (threadIdx.x == 0) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQ)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
     for (int t = 0; t < kQTiles; ++t) mbar_init(&bars->q_full[t], 1);
     mbar_init(&bars->q_empty, kQTiles);   // one commit per MMA issuer
     for (int s = 0; s < C::kStages; ++s) {
@@ -436,6 +440,9 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
+  // Q and K may come from the kernel before this one on the stream; tensor
+  // memory is only taken once that kernel has finished
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_u32(&bars->tmem_base)),
@@ -447,14 +454,13 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
   tc_fence_after();
   const uint32_t tmem = bars->tmem_base;
   volatile int* abort_flag = &bars->abort;
-  // the merge kernel may be scheduled now; it waits for this grid to finish
-  if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  // the merge kernel may be scheduled now (it waits for this grid to
+  // finish); a softmax thread signals it, keeping the producer free
+  if (threadIdx.x == 64) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (warp == 0) {
     // ------------------------------------------------------ TMA producer --
     if (lane == 0) {
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQ)) : "memory");
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
       bool ok = true;
       int li = 0;
       int sg = 0;
@@ -463,7 +469,9 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
         const Segment seg = segment_at(it, it_end, p.n_kt);
         const int bh = seg.u / p.n_qp, qp = seg.u - bh * p.n_qp;
         const int b = bh / p.H, h = bh - b * p.H;
-        ok = mbar_wait_bounded(&bars->q_empty, (uint32_t)((sg & 1) ^ 1), abort_flag, p.status);
+        // the Q buffer is free at the start; later segments wait for the
+        // MMAs of the previous one
+        if (sg > 0) ok = mbar_wait_bounded(&bars->q_empty, (uint32_t)((sg & 1) ^ 1), abort_flag, p.status);
         if (!ok) break;
         ++sg;   // Q of this segment is being issued
         q_armed = 0;
@@ -476,6 +484,13 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
             for (int cb = 0; cb < C::kCB; ++cb)
               tma_load_4d(sQ + t * C::kTileBytes + cb * (kBM * 128), &tmQ, cb * 64,
                           qp * kUnitRows + t * kBM, h, b, &bars->q_full[t]);
+          }
+          if (li == 1) {
+            // cold start: the first K tile lands before the rest of the ring
+            // is requested, so the first MMAs do not wait behind every
+            // CTA's whole prologue in HBM
+            ok = mbar_wait_bounded(&bars->k_full[0], 0, abort_flag, p.status);
+            if (!ok) break;
           }
           const int stage = (int)(li % C::kStages);
           const uint32_t ph = (uint32_t)((li / C::kStages) & 1);
@@ -623,6 +638,8 @@ constexpr int kFinRows = 32, kFinHeads = 32;
 __global__ void __launch_bounds__(kFinRows * kFinHeads)
 spatial_finalize_kernel(const TcParams p) {
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  // the main grid has completed: the next kernel may start its prologue
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   __shared__ float mass_s[kFinHeads][kFinRows + 1];
   const int r = threadIdx.x % kFinRows, hl = threadIdx.x / kFinRows;
   const int row_g = blockIdx.x * kFinRows + r;            // over B * n_qp * 256
