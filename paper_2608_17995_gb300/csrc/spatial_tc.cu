@@ -120,11 +120,26 @@ __device__ __forceinline__ uint64_t sw128_desc(const void* p) {
          ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
 
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t acc) {
+// The same descriptor as two 32-bit words: the low word holds the start
+// address (bits 0-13, in 16-byte units) and the leading-byte offset, the high
+// word the stride, version and swizzle fields, which are equal for every tile.
+// A K-step moves the start address only (no carry: shared memory < 256 KB), so
+// the issuer adds constants to the low word instead of rebuilding descriptors.
+__device__ __forceinline__ uint32_t sw128_desc_lo(const void* p) {
+  return (uint32_t)sw128_desc(p);
+}
+__device__ __forceinline__ uint32_t sw128_desc_hi() {
+  return (uint32_t)(((uint64_t)(1024 >> 4) << 32 | ((uint64_t)1 << 46) | ((uint64_t)2 << 61)) >> 32);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint32_t a_lo, uint32_t b_lo,
+                                         uint32_t hi, uint32_t acc) {
   asm volatile(
-      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a), "l"(b), "r"(kIdesc), "r"(acc));
+      "{\n\t.reg .pred p;\n\t.reg .b64 ad, bd;\n\t"
+      "setp.ne.b32 p, %5, 0;\n\t"
+      "mov.b64 ad, {%1, %3};\n\tmov.b64 bd, {%2, %3};\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %4, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_lo), "r"(b_lo), "r"(hi), "r"(kIdesc), "r"(acc));
 }
 
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
@@ -534,7 +549,12 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
       bool ok = true;
       int li = 0;
       int sg = 0;
-      const uint8_t* qa = sQ + t * C::kTileBytes;
+      // operand descriptors computed once; per MMA only constant offsets are
+      // added (the issuing thread shares its sub-partition with four busy
+      // softmax warps, so every instruction it needs delays the MMAs)
+      const uint32_t a_lo = sw128_desc_lo(sQ + t * C::kTileBytes);
+      const uint32_t b_lo0 = sw128_desc_lo(sK);
+      const uint32_t d_hi = sw128_desc_hi();
       const uint32_t d_base = tmem + (uint32_t)(t * 2 * kBN);
       for (int it = it_begin; it < it_end && ok;) {
         const Segment seg = segment_at(it, it_end, p.n_kt);
@@ -553,11 +573,11 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
           if (!ok) break;
           tc_fence_after();
           const uint32_t d_tmem = d_base + (uint32_t)(sb * kBN);
-          const uint8_t* kb = sK + stage * C::kTileBytes;
+          const uint32_t b_lo = b_lo0 + (uint32_t)((stage * C::kTileBytes) >> 4);
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
-            const int off = (kk >> 2) * (kBM * 128) + (kk & 3) * 32;
-            mma_bf16(d_tmem, sw128_desc(qa + off), sw128_desc(kb + off), kk > 0 ? 1u : 0u);
+            const uint32_t off = (uint32_t)(((kk >> 2) * (kBM * 128) + (kk & 3) * 32) >> 4);
+            mma_bf16(d_tmem, a_lo + off, b_lo + off, d_hi, kk > 0 ? 1u : 0u);
           }
           mma_commit(&bars->s_full[t][sb]);
           mma_commit(&bars->k_empty[stage]);
