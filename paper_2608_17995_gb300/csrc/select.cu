@@ -1,6 +1,7 @@
 // select.cu — joint score and token selection (Sec. 3.3.3, Eq. 8-9).
 //
-// One CTA of 512 threads per batch element, few barriers:
+// One CTA per batch element (256 threads up to M = 1024, 512 beyond; up to 8
+// keys per thread in registers), few barriers:
 //   1. min / max of A and V (NaN ignored): warp shuffles, one shared-memory
 //      round, every warp finishes the reduction itself;
 //   2. S = (alpha * A^) + ((1 - alpha) * V^) with explicitly rounded fp32
@@ -27,8 +28,7 @@
 namespace avits {
 namespace {
 
-constexpr int kThreads = 512;
-constexpr int kWarps = kThreads / 32;
+constexpr int kMaxThreads = 512;
 constexpr int kMaxRegKeys = 8;   // keys per thread kept in registers (M <= 4096)
 
 __device__ __forceinline__ uint32_t order_key(float s) {
@@ -58,12 +58,13 @@ __device__ __forceinline__ uint32_t count_digits(uint32_t key, bool valid, uint3
 
 // kRegKeys keys per thread in registers when M <= kRegKeys * kThreads; larger
 // M (kRegKeys = 0) keeps them in shared memory only.
-template <int kRegKeys>
+template <int kThreads, int kRegKeys>
 __global__ void __launch_bounds__(kThreads)
 fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V, int M, float alpha,
                    float eps, int k, float* __restrict__ S_out, int32_t* __restrict__ sel_idx,
                    uint8_t* __restrict__ mask, int32_t* __restrict__ tok_offset,
                    unsigned int* status) {
+  constexpr int kWarps = kThreads / 32;
   extern __shared__ uint32_t keys[];
   __shared__ float red[4][kWarps];
   __shared__ uint32_t cnt[2][kWarps][16];
@@ -276,27 +277,41 @@ cudaError_t launch_fuse_select(const float* A, const float* V, int B, int M, flo
     if (e != cudaSuccess) return e;
     if (!(dev >= 0 && dev < 64 && __atomic_load_n(&done[dev], __ATOMIC_ACQUIRE))) {
       const int mx = (int)(kSelectMaxM * sizeof(uint32_t));
-      e = cudaFuncSetAttribute(fuse_select_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+      e = cudaFuncSetAttribute(fuse_select_kernel<kMaxThreads, 0>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
       if (e != cudaSuccess) return e;
-      e = cudaFuncSetAttribute(fuse_select_kernel<kMaxRegKeys>,
+      e = cudaFuncSetAttribute(fuse_select_kernel<kMaxThreads, kMaxRegKeys>,
                                cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
       if (e != cudaSuccess) return e;
       if (dev >= 0 && dev < 64) __atomic_store_n(&done[dev], 1, __ATOMIC_RELEASE);
     }
   }
-  const int per = (M + kThreads - 1) / kThreads;
-  cudaError_t ce = prefer_max_shared<fuse_select_kernel<1>>();
-  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<2>>();
-  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<4>>();
-  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<kMaxRegKeys>>();
-  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<0>>();
+  // 256 threads up to M = 1024 (fewer warps to synchronise and scan over,
+  // measured faster at FLUX-1024), 512 beyond; shared memory only above 4096
+  void (*kern)(const float*, const float*, int, float, float, int, float*, int32_t*, uint8_t*,
+               int32_t*, unsigned int*);
+  int threads;
+  if (M <= 1024) {
+    threads = 256;
+    const int per = (M + 255) / 256;
+    kern = per <= 1   ? fuse_select_kernel<256, 1>
+           : per <= 2 ? fuse_select_kernel<256, 2>
+                      : fuse_select_kernel<256, 4>;
+  } else {
+    threads = kMaxThreads;
+    const int per = (M + kMaxThreads - 1) / kMaxThreads;
+    kern = per <= 4             ? fuse_select_kernel<kMaxThreads, 4>
+           : per <= kMaxRegKeys ? fuse_select_kernel<kMaxThreads, kMaxRegKeys>
+                                : fuse_select_kernel<kMaxThreads, 0>;
+  }
+  cudaError_t ce = prefer_max_shared<fuse_select_kernel<256, 1>>();
+  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<256, 2>>();
+  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<256, 4>>();
+  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<kMaxThreads, 4>>();
+  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<kMaxThreads, kMaxRegKeys>>();
+  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<kMaxThreads, 0>>();
   if (ce != cudaSuccess) return ce;
-  auto kern = per <= 1   ? fuse_select_kernel<1>
-              : per <= 2 ? fuse_select_kernel<2>
-              : per <= 4 ? fuse_select_kernel<4>
-              : per <= kMaxRegKeys ? fuse_select_kernel<kMaxRegKeys>
-                                   : fuse_select_kernel<0>;
-  cudaError_t e = launch_pdl(kern, dim3(B), dim3(kThreads), smem, s, A, V, M, alpha, eps, k, S,
+  cudaError_t e = launch_pdl(kern, dim3(B), dim3(threads), smem, s, A, V, M, alpha, eps, k, S,
                              sel_idx, mask, tok_offset, status);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
