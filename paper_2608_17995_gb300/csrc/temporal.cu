@@ -12,7 +12,9 @@
 //
 // avits_score_temporal_var: Eq. 6-7, unbiased variance over N_T snapshots
 // averaged over channels; two passes over the snapshot values held in
-// registers (mean, then squared deviations).
+// registers (mean, then squared deviations).  Main path: one CTA per token,
+// 16-byte loads, the N_T vectors of a position all issued before they are
+// reduced (HBM-bound: N_T * D * elt bytes per token).
 #include "avits_common.cuh"
 #include "avits_internal.h"
 
@@ -281,6 +283,79 @@ int grid_for(int64_t ntok, int num_sms) {
   return (int)(want < cap ? (want > 0 ? want : 1) : cap);
 }
 
+
+// Element e of a 16-byte vector, as fp32.
+template <typename T>
+__device__ __forceinline__ float vec_elem(const uint4& v, int e);
+template <>
+__device__ __forceinline__ float vec_elem<float>(const uint4& v, int e) {
+  const uint32_t w = e == 0 ? v.x : e == 1 ? v.y : e == 2 ? v.z : v.w;
+  return __uint_as_float(w);
+}
+template <>
+__device__ __forceinline__ float vec_elem<__nv_bfloat16>(const uint4& v, int e) {
+  const int q = e >> 1;
+  const uint32_t w = q == 0 ? v.x : q == 1 ? v.y : q == 2 ? v.z : v.w;
+  return (e & 1) ? bf16_hi(w) : bf16_lo(w);
+}
+
+// 16-byte vectors of kE elements; kNT >= n_t snapshots kept in registers.
+constexpr int kVarThreads = 128;
+
+template <typename T, int kNT>
+__global__ void __launch_bounds__(kVarThreads)
+temporal_var_vec_kernel(SnapPtrs snaps, int n_t, int64_t ntok, int D, float* __restrict__ V) {
+  constexpr int kE = 16 / (int)sizeof(T);
+  __shared__ float part[kVarThreads / 32];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int nv = D / kE;
+  const float inv_n = 1.0f / (float)n_t;
+  const float inv_n1 = 1.0f / (float)(n_t - 1);
+  for (int64_t t = blockIdx.x; t < ntok; t += gridDim.x) {
+    float acc = 0.f;
+    for (int v = threadIdx.x; v < nv; v += kVarThreads) {
+      uint4 raw[kNT];
+#pragma unroll
+      for (int s = 0; s < kNT; ++s)
+        if (s < n_t)
+          raw[s] = __ldcs(reinterpret_cast<const uint4*>(static_cast<const T*>(snaps.p[s]) +
+                                                        t * D) + v);
+#pragma unroll
+      for (int e = 0; e < kE; ++e) {
+        float z[kNT];
+        float mean = 0.f;
+#pragma unroll
+        for (int s = 0; s < kNT; ++s) {
+          if (s < n_t) {
+            z[s] = vec_elem<T>(raw[s], e);
+            mean += z[s];
+          }
+        }
+        mean *= inv_n;
+        float ss = 0.f;
+#pragma unroll
+        for (int s = 0; s < kNT; ++s) {
+          if (s < n_t) {
+            const float dv = z[s] - mean;
+            ss = fmaf(dv, dv, ss);
+          }
+        }
+        acc += ss * inv_n1;
+      }
+    }
+    acc = warp_sum(acc);
+    if (lane == 0) part[w] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      float tot = 0.f;
+#pragma unroll
+      for (int k = 0; k < kVarThreads / 32; ++k) tot += part[k];
+      V[t] = tot / (float)D;
+    }
+    __syncthreads();   // part[] is reused by the next token
+  }
+}
+
 }  // namespace
 
 template <typename T, bool kOverlapped = false>
@@ -395,6 +470,32 @@ cudaError_t launch_temporal_var(const void* const* snaps, int n_t, avits_dtype d
   SnapPtrs sp{};
   for (int i = 0; i < n_t; ++i) sp.p[i] = snaps[i];
   const int64_t ntok = (int64_t)B * N;
+  const int elt = (dt == AVITS_BF16) ? 2 : 4;
+  bool vec = ((int64_t)D * elt) % 16 == 0;
+  for (int i = 0; i < n_t; ++i) vec = vec && (reinterpret_cast<uintptr_t>(snaps[i]) & 15u) == 0;
+  if (vec) {
+    // one CTA per token (grid-stride beyond 2^31 - 1 tokens).  A plain
+    // launch: as a programmatic dependent its waiting CTAs took SM slots from
+    // the kernel before it and measured slower.
+    const unsigned grid = (unsigned)std::min<int64_t>(ntok, (int64_t)INT32_MAX);
+    if (dt == AVITS_BF16) {
+      if (n_t <= 4)
+        temporal_var_vec_kernel<__nv_bfloat16, 4><<<grid, kVarThreads, 0, s>>>(sp, n_t, ntok, D, V);
+      else if (n_t <= 8)
+        temporal_var_vec_kernel<__nv_bfloat16, 8><<<grid, kVarThreads, 0, s>>>(sp, n_t, ntok, D, V);
+      else
+        temporal_var_vec_kernel<__nv_bfloat16, kMaxSnapshots>
+            <<<grid, kVarThreads, 0, s>>>(sp, n_t, ntok, D, V);
+    } else {
+      if (n_t <= 4)
+        temporal_var_vec_kernel<float, 4><<<grid, kVarThreads, 0, s>>>(sp, n_t, ntok, D, V);
+      else if (n_t <= 8)
+        temporal_var_vec_kernel<float, 8><<<grid, kVarThreads, 0, s>>>(sp, n_t, ntok, D, V);
+      else
+        temporal_var_vec_kernel<float, kMaxSnapshots><<<grid, kVarThreads, 0, s>>>(sp, n_t, ntok, D, V);
+    }
+    return cudaGetLastError();
+  }
   const int grid = grid_for(ntok, num_sms);
   if (dt == AVITS_BF16)
     temporal_var_kernel<__nv_bfloat16><<<grid, kWarpsPerCta * 32, 0, s>>>(sp, n_t, ntok, D, V);

@@ -217,12 +217,16 @@ def test_temporal_odd_widths(av, orc, dtype, D):
     np.testing.assert_allclose(_np(V), orc.score_temporal(ht, hp), rtol=rtol, atol=1e-7)
 
 
-@pytest.mark.parametrize("dtype,n_t", [("f32", 2), ("f32", 5), ("bf16", 3)])
-def test_temporal_variance_eq7(av, orc, dtype, n_t):
+@pytest.mark.parametrize("dtype,n_t,D", [("f32", 2, 96), ("f32", 5, 96), ("bf16", 3, 96),
+                                         ("bf16", 4, 3072), ("bf16", 8, 200), ("f32", 12, 64),
+                                         ("bf16", 16, 40), ("bf16", 3, 30), ("f32", 6, 7)])
+def test_temporal_variance_eq7(av, orc, dtype, n_t, D):
+    """Eq. 6-7 over n_t snapshots: the 16-byte vector path (4, 8 and 16
+    snapshot variants) and the scalar path (rows not a multiple of 16 bytes)."""
     import torch
     from paper_2608_17995_gb300.workloads import to_bf16_bits
-    rng = np.random.default_rng(n_t)
-    B, N, D = 2, 50, 96
+    rng = np.random.default_rng(n_t + D)
+    B, N = 2, 50
     snaps = [rng.standard_normal((B, N, D)).astype(np.float32) for _ in range(n_t)]
     if dtype == "bf16":
         snaps = [to_bf16_bits(s) for s in snaps]
