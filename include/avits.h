@@ -213,6 +213,22 @@ avits_status avits_fuse_select(const float* A, const float* V, int B, int M, flo
                                uint8_t* sel_mask_opt, int32_t* tok_offset, void* stream);
 
 /* ------------------------------------------------------------------------
+ * avits_fuse_select with the paper's tie-breaking perturbation, Eq. 9
+ * (Sec. 3.3.3: small Gaussian noise added to the joint score before TopK).
+ * The noise is SUPPLIED BY THE CALLER (this library draws no random
+ * numbers):
+ *   S' = S + perturb   (one more rounded fp32 addition, after Eq. 8)
+ * and the selection is taken on S' (ties in S' still go to the lower index).
+ * perturb : NULL (exactly avits_fuse_select) or [B,M] fp32 device memory,
+ *           e.g. 1e-6 * N(0,1) per token as in the paper.
+ * S_opt receives S'.  Everything else as avits_fuse_select.
+ * ---------------------------------------------------------------------- */
+avits_status avits_fuse_select_perturbed(const float* A, const float* V, const float* perturb,
+                                         int B, int M, float alpha, float eps_norm, int k,
+                                         float* S_opt, int32_t* sel_idx, uint8_t* sel_mask_opt,
+                                         int32_t* tok_offset, void* stream);
+
+/* ------------------------------------------------------------------------
  * Selective upsampling, Sec. 3.2 Stage 2: selected tokens are expanded to
  * the next resolution, the others stay as they are, and all of them go into
  * one packed mixed-resolution sequence of N_out = M + 3k tokens.

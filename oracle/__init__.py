@@ -139,14 +139,18 @@ def score_temporal_var(snaps: Sequence[np.ndarray]) -> np.ndarray:
     return V
 
 
-def fuse(A: np.ndarray, V: np.ndarray, alpha: float, eps: float = 1e-6) -> np.ndarray:
+def fuse(A: np.ndarray, V: np.ndarray, alpha: float, eps: float = 1e-6,
+         perturb: Optional[np.ndarray] = None) -> np.ndarray:
+    """Min-max normalisation and Eq. 8; with ``perturb`` the caller's
+    tie-breaking noise of Eq. 9 is added to S (one rounded fp32 addition)."""
     lib = _load()
     A = _c(np.asarray(A, np.float32))
     V = _c(np.asarray(V, np.float32))
     B, M = A.shape
+    P = None if perturb is None else _c(np.asarray(perturb, np.float32).reshape(B, M))
     S = np.zeros((B, M), np.float32)
     rc = lib.avits_oracle_fuse(_p(A), _p(V), B, M, ctypes.c_float(alpha), ctypes.c_float(eps),
-                               _p(S))
+                               _p(P), _p(S))
     if rc != 0:
         raise ValueError("oracle fuse: bad arguments")
     return S
@@ -166,8 +170,8 @@ def topk(S: np.ndarray, k: int):
     return sel, mask, off
 
 
-def fuse_select(A, V, alpha: float, k: int, eps: float = 1e-6):
-    S = fuse(A, V, alpha, eps)
+def fuse_select(A, V, alpha: float, k: int, eps: float = 1e-6, perturb=None):
+    S = fuse(A, V, alpha, eps, perturb)
     sel, mask, off = topk(S, k)
     return S, sel, mask, off
 

@@ -200,8 +200,11 @@ static void minmax_f32(const float* x, int M, float* mn, float* mx) {
   *mx = hi;
 }
 
+/* perturb (NULL or [B,M]): the paper's tie-breaking noise, Eq. 9 (Sec.
+ * 3.3.3), supplied by the caller and added to S as one more rounded fp32
+ * addition: S' = S + perturb. */
 int avits_oracle_fuse(const float* A, const float* V, int B, int M, float alpha, float eps,
-                      float* S) {
+                      const float* perturb, float* S) {
   if (B <= 0 || M <= 0) return OR_BAD_ARG;
   for (int b = 0; b < B; ++b) {
     const float* a = A + (int64_t)b * M;
@@ -221,7 +224,9 @@ int avits_oracle_fuse(const float* A, const float* V, int B, int M, float alpha,
       vn = vn / vden;
       volatile float t1 = alpha * an;
       volatile float t2 = one_m * vn;
-      S[(int64_t)b * M + i] = t1 + t2;
+      volatile float sc = t1 + t2;
+      if (perturb) sc = sc + perturb[(int64_t)b * M + i];
+      S[(int64_t)b * M + i] = sc;
     }
   }
   return OR_OK;

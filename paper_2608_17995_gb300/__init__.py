@@ -76,6 +76,7 @@ def lib():
                                        f32, vp, vp],
         "avits_score_temporal_var": [vp, i32, i32, i32, i32, i32, vp, vp],
         "avits_fuse_select": [vp, vp, i32, i32, f32, f32, i32, vp, vp, vp, vp, vp],
+        "avits_fuse_select_perturbed": [vp, vp, vp, i32, i32, f32, f32, i32, vp, vp, vp, vp, vp],
         "avits_selective_upsample": [vp, i32, i32, i32, i32, i32, i32, i32, vp, vp, vp, vp, i32,
                                      i32, vp, vp, vp, vp, vp, vp],
         "avits_merge_final": [vp, i32, i32, i32, vp, vp, i32, i32, i32, i32, i32, vp, vp, sz, vp],
@@ -257,12 +258,23 @@ def avits_score_temporal_var(snaps: Sequence, V, stream=None):
 
 
 def avits_fuse_select(A, V, alpha: float, k: int, sel_idx, tok_offset, S=None, sel_mask=None,
-                      eps_norm: float = 1e-6, stream=None):
+                      eps_norm: float = 1e-6, stream=None, perturb=None):
+    """Eq. 8-9; ``perturb`` ([B,M] fp32, optional): the caller's tie-breaking
+    noise, added to S before the selection (avits_fuse_select_perturbed)."""
     B, M = A.shape
-    rc = lib().avits_fuse_select(_ptr(A), _ptr(V), B, M, float(alpha), float(eps_norm), int(k),
-                                 _ptr(S), _ptr(sel_idx), _ptr(sel_mask), _ptr(tok_offset),
-                                 _stream(stream))
-    _check("avits_fuse_select", rc)
+    if perturb is None:
+        rc = lib().avits_fuse_select(_ptr(A), _ptr(V), B, M, float(alpha), float(eps_norm),
+                                     int(k), _ptr(S), _ptr(sel_idx), _ptr(sel_mask),
+                                     _ptr(tok_offset), _stream(stream))
+        _check("avits_fuse_select", rc)
+    else:
+        if tuple(perturb.shape) != (B, M):
+            raise ValueError("perturb must be [B,M]")
+        rc = lib().avits_fuse_select_perturbed(_ptr(A), _ptr(V), _ptr(perturb), B, M,
+                                               float(alpha), float(eps_norm), int(k), _ptr(S),
+                                               _ptr(sel_idx), _ptr(sel_mask), _ptr(tok_offset),
+                                               _stream(stream))
+        _check("avits_fuse_select_perturbed", rc)
     return sel_idx
 
 

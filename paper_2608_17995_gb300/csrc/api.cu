@@ -166,10 +166,18 @@ avits_status avits_score_temporal_var(const void* const* snaps, int n_t, avits_d
 avits_status avits_fuse_select(const float* A, const float* V, int B, int M, float alpha,
                                float eps_norm, int k, float* S_opt, int32_t* sel_idx,
                                uint8_t* sel_mask_opt, int32_t* tok_offset, void* stream) {
+  return avits_fuse_select_perturbed(A, V, nullptr, B, M, alpha, eps_norm, k, S_opt, sel_idx,
+                                     sel_mask_opt, tok_offset, stream);
+}
+
+avits_status avits_fuse_select_perturbed(const float* A, const float* V, const float* perturb,
+                                         int B, int M, float alpha, float eps_norm, int k,
+                                         float* S_opt, int32_t* sel_idx, uint8_t* sel_mask_opt,
+                                         int32_t* tok_offset, void* stream) {
   if (!A || !V || !tok_offset || (k > 0 && !sel_idx)) return AVITS_ERR_INVALID_ARG;
   if (B <= 0 || M <= 0 || M > kSelectMaxM || k < 0 || k > M) return AVITS_ERR_INVALID_ARG;
   if (!(alpha >= 0.f && alpha <= 1.f) || !(eps_norm >= 0.f)) return AVITS_ERR_INVALID_ARG;
-  return cuda_status(launch_fuse_select(A, V, B, M, alpha, eps_norm, k, S_opt, sel_idx,
+  return cuda_status(launch_fuse_select(A, V, perturb, B, M, alpha, eps_norm, k, S_opt, sel_idx,
                                         sel_mask_opt, tok_offset, status_word(),
                                         static_cast<cudaStream_t>(stream)));
 }

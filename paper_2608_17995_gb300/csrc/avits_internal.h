@@ -55,9 +55,10 @@ cudaError_t launch_temporal_var(const void* const* snaps, int n_t, avits_dtype d
 
 // ---- fuse + select (Eq. 8-9) ------------------------------------------------
 constexpr int kSelectMaxM = 32768;
-cudaError_t launch_fuse_select(const float* A, const float* V, int B, int M, float alpha,
-                               float eps, int k, float* S, int32_t* sel_idx, uint8_t* mask,
-                               int32_t* tok_offset, unsigned int* status, cudaStream_t s);
+cudaError_t launch_fuse_select(const float* A, const float* V, const float* perturb, int B, int M,
+                               float alpha, float eps, int k, float* S, int32_t* sel_idx,
+                               uint8_t* mask, int32_t* tok_offset, unsigned int* status,
+                               cudaStream_t s);
 
 // ---- selective upsample (Stage 2) -------------------------------------------
 cudaError_t launch_upsample(const void* latent, avits_dtype dt, int B, int M, int gh, int gw,

@@ -6,7 +6,9 @@
 //      round, every warp finishes the reduction itself;
 //   2. S = (alpha * A^) + ((1 - alpha) * V^) with explicitly rounded fp32
 //      operations in that order (no contraction), so that the same A, V give
-//      bit-identical S wherever the selection is recomputed; each S becomes
+//      bit-identical S wherever the selection is recomputed; with a
+//      caller-supplied perturbation (the tie-breaking noise of Eq. 9) one more
+//      rounded addition S + perturb follows; each S becomes
 //      an order-preserving 32-bit key (NaN -> 0, below everything; -0 -> +0;
 //      otherwise the IEEE bits with the sign bit flipped if positive, all
 //      bits flipped if negative), kept in registers and in shared memory;
@@ -60,7 +62,8 @@ __device__ __forceinline__ uint32_t count_digits(uint32_t key, bool valid, uint3
 // M (kRegKeys = 0) keeps them in shared memory only.
 template <int kThreads, int kRegKeys>
 __global__ void __launch_bounds__(kThreads)
-fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V, int M, float alpha,
+fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V,
+                   const float* __restrict__ perturb, int M, float alpha,
                    float eps, int k, float* __restrict__ S_out, int32_t* __restrict__ sel_idx,
                    uint8_t* __restrict__ mask, int32_t* __restrict__ tok_offset,
                    unsigned int* status) {
@@ -76,6 +79,7 @@ fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V, int
   const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   const float* a = A + (int64_t)b * M;
   const float* v = V + (int64_t)b * M;
+  const float* pt = perturb ? perturb + (int64_t)b * M : nullptr;
   constexpr bool in_regs = kRegKeys > 0;
   constexpr int R = kRegKeys > 0 ? kRegKeys : 1;
 
@@ -133,10 +137,11 @@ fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V, int
   const float one_m = __fsub_rn(1.0f, alpha);
   int any_nan = 0;
   uint32_t rk[R];
-  auto fuse = [&](float x, float y) {
+  auto fuse = [&](float x, float y, int i) {
     const float an = __fdiv_rn(__fsub_rn(x, amn), aden);
     const float vn = __fdiv_rn(__fsub_rn(y, vmn), vden);
-    return __fadd_rn(__fmul_rn(alpha, an), __fmul_rn(one_m, vn));
+    const float sc = __fadd_rn(__fmul_rn(alpha, an), __fmul_rn(one_m, vn));
+    return pt ? __fadd_rn(sc, pt[i]) : sc;
   };
   if (in_regs) {
 #pragma unroll
@@ -144,7 +149,7 @@ fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V, int
       const int i = tid + r * kThreads;
       rk[r] = 0u;
       if (i < M) {
-        const float s = fuse(ra[r], rv[r]);
+        const float s = fuse(ra[r], rv[r], i);
         if (S_out) S_out[(int64_t)b * M + i] = s;
         any_nan |= (s != s);
         rk[r] = order_key(s);
@@ -153,7 +158,7 @@ fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V, int
     }
   } else {
     for (int i = tid; i < M; i += kThreads) {
-      const float s = fuse(a[i], v[i]);
+      const float s = fuse(a[i], v[i], i);
       if (S_out) S_out[(int64_t)b * M + i] = s;
       any_nan |= (s != s);
       keys[i] = order_key(s);
@@ -265,9 +270,10 @@ fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V, int
 
 }  // namespace
 
-cudaError_t launch_fuse_select(const float* A, const float* V, int B, int M, float alpha,
-                               float eps, int k, float* S, int32_t* sel_idx, uint8_t* mask,
-                               int32_t* tok_offset, unsigned int* status, cudaStream_t s) {
+cudaError_t launch_fuse_select(const float* A, const float* V, const float* perturb, int B, int M,
+                               float alpha, float eps, int k, float* S, int32_t* sel_idx,
+                               uint8_t* mask, int32_t* tok_offset, unsigned int* status,
+                               cudaStream_t s) {
   const size_t smem = (size_t)M * sizeof(uint32_t);
   if (smem > 48 * 1024) {
     // opt in once per device to the largest size any call can ask for
@@ -288,8 +294,8 @@ cudaError_t launch_fuse_select(const float* A, const float* V, int B, int M, flo
   }
   // 256 threads up to M = 1024 (fewer warps to synchronise and scan over,
   // measured faster at FLUX-1024), 512 beyond; shared memory only above 4096
-  void (*kern)(const float*, const float*, int, float, float, int, float*, int32_t*, uint8_t*,
-               int32_t*, unsigned int*);
+  void (*kern)(const float*, const float*, const float*, int, float, float, int, float*,
+               int32_t*, uint8_t*, int32_t*, unsigned int*);
   int threads;
   if (M <= 1024) {
     threads = 256;
@@ -311,8 +317,8 @@ cudaError_t launch_fuse_select(const float* A, const float* V, int B, int M, flo
   if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<kMaxThreads, kMaxRegKeys>>();
   if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<kMaxThreads, 0>>();
   if (ce != cudaSuccess) return ce;
-  cudaError_t e = launch_pdl(kern, dim3(B), dim3(threads), smem, s, A, V, M, alpha, eps, k, S,
-                             sel_idx, mask, tok_offset, status);
+  cudaError_t e = launch_pdl(kern, dim3(B), dim3(threads), smem, s, A, V, perturb, M, alpha, eps,
+                             k, S, sel_idx, mask, tok_offset, status);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

@@ -237,6 +237,41 @@ def test_temporal_variance_eq7(av, orc, dtype, n_t, D):
 
 # ---------------------------------------------------------- fuse/select ----
 
+
+@pytest.mark.parametrize("M,k,ties", [(1024, 307, True), (3000, 900, False), (9000, 2000, True)])
+def test_fuse_select_perturbed_bitexact(av, orc, M, k, ties):
+    """Eq. 9 with caller-supplied tie-breaking noise: S' and the selection
+    bit-exact against the oracle (register and shared-memory key paths)."""
+    import torch
+    from paper_2608_17995_gb300.workloads import random_scores
+    A, V = random_scores(40 + M, 2, M, ties=ties)
+    rng = np.random.default_rng(M)
+    d = (1e-6 * rng.standard_normal((2, M))).astype(np.float32)
+    S_o = orc.fuse(A, V, 0.5, perturb=d)
+    sel_o, mask_o, off_o = orc.topk(S_o, k)
+    dev = lambda x: torch.from_numpy(np.ascontiguousarray(x)).cuda()
+    S = torch.empty(2, M, dtype=torch.float32, device="cuda")
+    sel = torch.empty(2, k, dtype=torch.int32, device="cuda")
+    mask = torch.empty(2, M, dtype=torch.uint8, device="cuda")
+    off = torch.empty(2, M, dtype=torch.int32, device="cuda")
+    av.avits_fuse_select(dev(A), dev(V), 0.5, k, sel, off, S=S, sel_mask=mask, perturb=dev(d))
+    assert np.array_equal(_np(S).view(np.uint32), S_o.view(np.uint32))
+    assert np.array_equal(_np(sel), sel_o)
+    assert np.array_equal(_np(mask), mask_o)
+    assert np.array_equal(_np(off), off_o)
+    # zero noise: exactly the unperturbed call
+    S2 = torch.empty_like(S)
+    sel2 = torch.empty_like(sel)
+    off2 = torch.empty_like(off)
+    av.avits_fuse_select(dev(A), dev(V), 0.5, k, sel2, off2, S=S2,
+                         perturb=torch.zeros(2, M, dtype=torch.float32, device="cuda"))
+    S3 = torch.empty_like(S)
+    sel3 = torch.empty_like(sel)
+    off3 = torch.empty_like(off)
+    av.avits_fuse_select(dev(A), dev(V), 0.5, k, sel3, off3, S=S3)
+    assert torch.equal(S2.view(torch.int32), S3.view(torch.int32))
+    assert torch.equal(sel2, sel3) and torch.equal(off2, off3)
+
 def _run_select(av, A, V, alpha, k):
     import torch
     B, M = A.shape

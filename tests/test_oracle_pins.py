@@ -200,6 +200,29 @@ def test_fuse_alpha_arms_and_range(oracle_mod):
     np.testing.assert_allclose(Sc, 0.5 * oracle_mod.fuse(V[:1, :10], V[:1, :10], 1.0), rtol=1e-6)
 
 
+def test_perturbation_breaks_ties_and_is_one_rounded_add(oracle_mod):
+    """Eq. 9's tie-breaking noise (caller-supplied): zero noise is the plain
+    selection bit for bit; +1e-6 on one of three tied tokens moves it ahead
+    of the others (a dropped or sign-flipped term keeps the lower-index
+    tokens); S' - S equals the noise to within half an ulp of S'."""
+    A = np.array([[0.5, 0.9, 0.5, 0.5, 0.1]], np.float32)
+    V = np.zeros_like(A)
+    S0 = oracle_mod.fuse(A, V, 1.0)
+    Sz = oracle_mod.fuse(A, V, 1.0, perturb=np.zeros_like(A))
+    assert np.array_equal(S0.view(np.uint32), Sz.view(np.uint32))
+    assert oracle_mod.topk(S0, 3)[0][0].tolist() == [0, 1, 2]
+    d = np.array([[0.0, 0.0, 0.0, 1e-6, 0.0]], np.float32)
+    S1 = oracle_mod.fuse(A, V, 1.0, perturb=d)
+    assert oracle_mod.topk(S1, 3)[0][0].tolist() == [0, 1, 3]
+    rng = np.random.default_rng(5)
+    Ar, Vr = rng.random((2, 300), dtype=np.float32), rng.random((2, 300), dtype=np.float32)
+    dr = (1e-6 * rng.standard_normal((2, 300))).astype(np.float32)
+    Sa = oracle_mod.fuse(Ar, Vr, 0.5).astype(np.float64)
+    Sb = oracle_mod.fuse(Ar, Vr, 0.5, perturb=dr)
+    err = np.abs(Sb.astype(np.float64) - Sa - dr.astype(np.float64))
+    assert np.all(err <= 0.5 * np.spacing(Sb).astype(np.float64))
+
+
 @pytest.mark.parametrize("seed,M,k,ties", [(0, 50, 7, False), (1, 300, 300, True),
                                             (2, 1000, 0, True), (3, 1024, 307, True),
                                             (4, 1, 1, False)])
