@@ -76,11 +76,13 @@ def score_spatial(q_img: np.ndarray, k_all: np.ndarray, L: int, softmax_scale: f
                   weight: float = 1.0, A_in: Optional[np.ndarray] = None,
                   rows: Optional[Sequence[int]] = None, l2norm: bool = False,
                   q_strides: Optional[Sequence[int]] = None,
-                  k_strides: Optional[Sequence[int]] = None, shape=None):
+                  k_strides: Optional[Sequence[int]] = None, shape=None,
+                  text_mask: Optional[np.ndarray] = None):
     """Eq. 3 / Eq. 5.  q_img [B,H,M,d], k_all [B,H,Nk,d] (or flat buffers with
     explicit element strides and shape=(B,H,M,Nk,d)).  Returns (A [B,M] fp32,
     mass [B,H,M] fp64, lse [B,H,M,2] fp64); with ``rows`` only those flat
-    b*M+i entries are computed (others are 0)."""
+    b*M+i entries are computed (others are 0).  ``text_mask`` ([B,Nk], nonzero
+    = text key) replaces the first-L rule for interleaved sequences."""
     lib = _load()
     dt = _dtype_code(q_img)
     if _dtype_code(k_all) != dt:
@@ -98,6 +100,9 @@ def score_spatial(q_img: np.ndarray, k_all: np.ndarray, L: int, softmax_scale: f
     mass = np.zeros((B, H, M), np.float64)
     lse = np.zeros((B, H, M, 2), np.float64)
     rows_arr = None if rows is None else np.ascontiguousarray(np.asarray(rows, np.int32))
+    tm = None
+    if text_mask is not None:
+        tm = np.ascontiguousarray((np.asarray(text_mask) != 0).astype(np.uint8).reshape(B, Nk))
     fn = lib.avits_oracle_score_spatial
     fn.restype = ctypes.c_int
     i64 = ctypes.c_int64
@@ -106,7 +111,8 @@ def score_spatial(q_img: np.ndarray, k_all: np.ndarray, L: int, softmax_scale: f
             i64(k_strides[0]), i64(k_strides[1]), i64(k_strides[2]),
             ctypes.c_double(softmax_scale), ctypes.c_double(weight),
             0 if A_in is None else 1, 1 if l2norm else 0,
-            _p(rows_arr), 0 if rows_arr is None else len(rows_arr), _p(A), _p(mass), _p(lse))
+            _p(rows_arr), 0 if rows_arr is None else len(rows_arr), _p(tm), _p(A), _p(mass),
+            _p(lse))
     if rc != 0:
         raise ValueError("oracle score_spatial: bad arguments (%d)" % rc)
     return A, mass, lse

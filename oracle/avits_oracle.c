@@ -80,12 +80,17 @@ static void put_elem(void* base, int dtype, int64_t idx, float v) {
  *
  * rows: NULL for all B*M queries, else `nrows` flat indices b*M + i.
  * mass_out [B,H,M] and lse_out [B,H,M,2] are optional (fp64).
+ * text_mask: NULL (the text keys are the first L), else [B,Nk] bytes, key j
+ * of element b is a text key iff text_mask[b*Nk + j] != 0 (the unified
+ * sequences of MLLM-conditioned models, where text and image tokens
+ * interleave; Sec. 3.3.1).  L is then ignored.
  * ------------------------------------------------------------------------- */
 int avits_oracle_score_spatial(const void* q, const void* k, int dtype, int B, int H, int M,
                                int Nk, int L, int d, int64_t q_sb, int64_t q_sh, int64_t q_sn,
                                int64_t k_sb, int64_t k_sh, int64_t k_sn, double scale,
                                double weight, int accumulate, int l2norm, const int32_t* rows,
-                               int nrows, float* A, double* mass_out, double* lse_out) {
+                               int nrows, const uint8_t* text_mask, float* A, double* mass_out,
+                               double* lse_out) {
   if (B <= 0 || H <= 0 || M <= 0 || Nk <= 0 || d <= 0 || L < 0 || L > Nk) return OR_BAD_ARG;
   int n = rows ? nrows : B * M;
   int bad = 0;
@@ -120,7 +125,10 @@ int avits_oracle_score_spatial(const void* q, const void* k, int dtype, int B, i
       double z = 0.0;
       for (int j = 0; j < Nk; ++j) { P[j] = exp(P[j] - mx); z += P[j]; }
       double mass = 0.0, ztxt = 0.0;
-      for (int j = 0; j < L; ++j) { mass += P[j] / z; ztxt += P[j]; }   /* image->text block */
+      for (int j = 0; j < Nk; ++j) {                                      /* image->text block */
+        const int is_text = text_mask ? text_mask[(int64_t)b * Nk + j] != 0 : j < L;
+        if (is_text) { mass += P[j] / z; ztxt += P[j]; }
+      }
       head_sum += mass;
       if (mass_out) mass_out[((int64_t)b * H + h) * M + i] = mass;
       if (lse_out) {

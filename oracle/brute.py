@@ -18,15 +18,20 @@ def as_f64(a: np.ndarray) -> np.ndarray:
     return bf16_to_f64(a) if a.dtype == np.uint16 else np.asarray(a, np.float64)
 
 
-def spatial_full_softmax(q_img, k_all, L, scale):
+def spatial_full_softmax(q_img, k_all, L, scale, text_mask=None):
     """A [B,M] and mass [B,H,M]: softmax(Q K^T * scale) over all keys
-    (scipy's softmax), text columns summed, mean over heads (Eq. 3)."""
+    (scipy's softmax), text columns summed, mean over heads (Eq. 3).  The
+    text columns are the first L, or those where text_mask [B,Nk] is set."""
     from scipy.special import softmax
     q = as_f64(q_img)
     k = as_f64(k_all)
     P = np.einsum("bhmd,bhnd->bhmn", q, k) * scale
     alpha = softmax(P, axis=-1)
-    mass = alpha[..., :L].sum(-1)
+    if text_mask is None:
+        mass = alpha[..., :L].sum(-1)
+    else:
+        w = (np.asarray(text_mask) != 0).astype(np.float64)[:, None, None, :]
+        mass = (alpha * w).sum(-1)
     return mass.mean(axis=1), mass
 
 

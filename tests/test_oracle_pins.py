@@ -135,6 +135,35 @@ def test_spatial_l2norm_reading_scale_invariant(oracle_mod):
 
 # --------------------------------------------------------------- temporal --
 
+@pytest.mark.parametrize("seed,B,H,M,Nk,d", [(0, 2, 3, 7, 40, 16), (1, 1, 2, 33, 97, 8)])
+def test_spatial_text_mask(oracle_mod, seed, B, H, M, Nk, d):
+    """Interleaved text keys (MLLM-style sequences): the masked oracle equals
+    the materialised softmax with the masked columns summed; a first-L mask
+    is the L form bit for bit; a mask and its complement add up to 1; moving
+    keys and mask together changes nothing."""
+    from oracle import brute
+    rng = np.random.default_rng(seed)
+    q = rng.standard_normal((B, H, M, d)).astype(np.float32)
+    k = rng.standard_normal((B, H, Nk, d)).astype(np.float32)
+    mask = (rng.random((B, Nk)) < 0.3).astype(np.uint8)
+    A, mass, _ = oracle_mod.score_spatial(q, k, 0, 0.4, text_mask=mask)
+    A_b, mass_b = brute.spatial_full_softmax(q, k, 0, 0.4, text_mask=mask)
+    np.testing.assert_allclose(mass, mass_b, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(A, A_b, rtol=1e-6, atol=1e-7)
+    L = Nk // 3
+    first = np.zeros((B, Nk), np.uint8)
+    first[:, :L] = 1
+    _, mass_l, lse_l = oracle_mod.score_spatial(q, k, L, 0.4)
+    _, mass_f, lse_f = oracle_mod.score_spatial(q, k, 0, 0.4, text_mask=first)
+    assert np.array_equal(mass_l, mass_f) and np.array_equal(lse_l, lse_f)
+    _, mass_c, _ = oracle_mod.score_spatial(q, k, 0, 0.4, text_mask=1 - mask)
+    np.testing.assert_allclose(mass + mass_c, 1.0, rtol=0, atol=1e-12)
+    perm = rng.permutation(Nk)
+    _, mass_p, _ = oracle_mod.score_spatial(q, np.ascontiguousarray(k[:, :, perm]), 0, 0.4,
+                                            text_mask=np.ascontiguousarray(mask[:, perm]))
+    np.testing.assert_allclose(mass_p, mass, rtol=0, atol=1e-12)
+
+
 def test_temporal_closed_forms(oracle_mod):
     """P2: h_t = c h_prev gives |c-1| |h| / (|h| + eps); h_prev = 0 gives |h_t|/eps."""
     rng = np.random.default_rng(1)
