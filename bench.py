@@ -360,6 +360,7 @@ def run_ours(args, world, rank, local, pg):
         result["warm_l2"] = warm_measure(torch, buf, sets, stream, K)
         result["batched_schedule"] = batched_schedule_measure(torch, av, dev, stream, K)
         result["temporal_var"] = temporal_var_measure(torch, av, tr, dev, stream, peaks)
+        result["spatial_keymask"] = keymask_measure(torch, av, buf, tr, sets, nsets, stream, peaks)
     return result, tr
 
 
@@ -484,6 +485,39 @@ def batched_schedule_measure(torch, av, dev, stream, K):
             "transitions_per_s": round(2 * t1.B * 1e3 / ms, 1), "status": st,
             "config": "B=8, FLUX heads/width, 16x16 -> 32x32 (k=128) -> 64x64 (k=192, 640 "
                       "mixed tokens re-scored), final merge; nearest"}
+
+
+def keymask_measure(torch, av, buf, tr, sets, nsets, stream, peaks):
+    """avits_score_spatial_keymask at the FLUX-1024 shape (interleaved text
+    and image keys): text blocks between image blocks (a unified MLLM-style
+    sequence; most key halves all text or all image) and a random 30 % mask
+    (every key half mixed, the slow path)."""
+    Nk = tr.Nk
+    g = torch.Generator(device="cpu")
+    g.manual_seed(3)
+    blocks = torch.zeros(tr.B, Nk, dtype=torch.uint8)
+    blocks[:, 0:200] = 1
+    blocks[:, 700:900] = 1
+    blocks[:, 1400:1512] = 1
+    rand = (torch.rand(tr.B, Nk, generator=g) < 0.3).to(torch.uint8)
+    A = torch.empty(tr.B, tr.M, dtype=torch.float32, device=buf.A.device)
+    out = {}
+    flops = 2.0 * tr.B * tr.H * tr.M * Nk * tr.d
+    for name, m in (("blocks", blocks), ("random", rand)):
+        md = m.to(buf.A.device)
+
+        def fn():
+            for s_ in range(nsets):
+                av.avits_score_spatial(sets[s_][0], sets[s_][1], 0, tr.softmax_scale, A,
+                                       workspace=buf.ws, stream=stream, text_mask=md)
+
+        ms = _graph_time_ms(torch, stream, fn, 20) / nsets
+        tf = flops / (ms * 1e-3) / 1e12
+        out[name] = {"us": round(ms * 1e3, 3), "tflops": round(tf, 2),
+                     "frac_tensor": round(tf / peaks["bf16_tflops"], 4),
+                     "text_keys": int(m.sum())}
+    out["status"] = av.avits_device_status(stream)
+    return out
 
 
 def temporal_var_measure(torch, av, tr, dev, stream, peaks, n_t=4, n_sets=6):

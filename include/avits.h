@@ -146,6 +146,22 @@ size_t avits_score_spatial_noalloc_limit(void);
 const char* avits_score_spatial_noalloc_error(void);
 
 /* ------------------------------------------------------------------------
+ * avits_score_spatial for sequences whose text and image tokens interleave
+ * (the unified sequences of MLLM-conditioned models, Sec. 3.3.1): the text
+ * keys are the keys j with text_mask[b*Nk + j] != 0 instead of the first L.
+ * text_mask : [B,Nk] uint8 device memory (one byte per key).  Everything else
+ * (Eq. 3-5, layouts, workspace, weight / accumulate, lse_opt) as
+ * avits_score_spatial; lse_opt[...,1] is the logsumexp over the masked keys.
+ * ---------------------------------------------------------------------- */
+avits_status avits_score_spatial_keymask(const void* q_img, const void* k_all, avits_dtype dt,
+                                         int B, int H, int M, int Nk, int d, int64_t q_sb,
+                                         int64_t q_sh, int64_t q_sn, int64_t k_sb, int64_t k_sh,
+                                         int64_t k_sn, const uint8_t* text_mask,
+                                         float softmax_scale, float weight, int accumulate,
+                                         float* A, float* lse_opt, void* workspace,
+                                         size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
  * Temporal importance.  Sec. 3.3.2 scores a token by how much its feature
  * moves across the collected denoising steps.  This call takes the two most
  * recent snapshots and returns the relative step change

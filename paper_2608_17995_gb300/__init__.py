@@ -70,6 +70,8 @@ def lib():
         "avits_score_spatial": [vp, vp, i32, i32, i32, i32, i32, i32, i32, i64, i64, i64, i64, i64,
                                 i64, f32, f32, i32, vp, vp, vp, sz, vp],
         "avits_score_spatial_workspace": [i32, i32, i32, i32, i32, i32],
+        "avits_score_spatial_keymask": [vp, vp, i32, i32, i32, i32, i32, i32, i64, i64, i64, i64,
+                                        i64, i64, vp, f32, f32, i32, vp, vp, vp, sz, vp],
         "avits_score_temporal": [vp, vp, i32, i32, i32, i32, f32, vp, vp],
         "avits_score_spatiotemporal": [vp, vp, i32, i32, i32, i32, i32, i32, i32, i64, i64, i64,
                                        i64, i64, i64, f32, f32, i32, vp, vp, vp, sz, vp, vp, i32,
@@ -181,9 +183,12 @@ _default_ws = {}
 
 def avits_score_spatial(q_img, k_all, L: int, softmax_scale: float, A, weight: float = 1.0,
                         accumulate: bool = False, lse=None, workspace: Optional[SpatialWorkspace] = None,
-                        stream=None):
+                        stream=None, text_mask=None):
     """Eq. 3-5.  q_img [B,H,M,d] (any strides, d contiguous), k_all [B,H,Nk,d]
-    with the L text keys first; A [B,M] fp32 written (or accumulated)."""
+    with the L text keys first; A [B,M] fp32 written (or accumulated).  With
+    ``text_mask`` ([B,Nk] uint8 / bool on the device, nonzero = text key) the
+    text keys are the masked ones instead (avits_score_spatial_keymask; L is
+    ignored)."""
     B, H, M, d = q_img.shape
     Nk = k_all.shape[2]
     if k_all.shape[0] != B or k_all.shape[1] != H or k_all.shape[3] != d:
@@ -198,6 +203,18 @@ def avits_score_spatial(q_img, k_all, L: int, softmax_scale: float, A, weight: f
         key = (q_img.device.index, _torch().cuda.current_stream().cuda_stream if stream is None else _stream(stream))
         workspace = _default_ws.setdefault(key, SpatialWorkspace(q_img.device))
     wbuf, wbytes = workspace.get(need)
+    if text_mask is not None:
+        if tuple(text_mask.shape) != (B, Nk) or text_mask.element_size() != 1 or \
+                not text_mask.is_contiguous():
+            raise ValueError("text_mask must be a contiguous [B,Nk] byte tensor")
+        rc = lib().avits_score_spatial_keymask(
+            _ptr(q_img), _ptr(k_all), dt, B, H, M, Nk, d,
+            q_img.stride(0), q_img.stride(1), q_img.stride(2),
+            k_all.stride(0), k_all.stride(1), k_all.stride(2), _ptr(text_mask),
+            float(softmax_scale), float(weight), 1 if accumulate else 0,
+            _ptr(A), _ptr(lse), _ptr(wbuf), wbytes, _stream(stream))
+        _check("avits_score_spatial_keymask", rc)
+        return A
     rc = lib().avits_score_spatial(
         _ptr(q_img), _ptr(k_all), dt, B, H, M, Nk, L, d,
         q_img.stride(0), q_img.stride(1), q_img.stride(2),

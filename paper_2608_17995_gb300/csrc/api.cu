@@ -110,6 +110,32 @@ avits_status avits_score_spatial(const void* q_img, const void* k_all, avits_dty
   return cuda_status(launch_spatial_simt(a, s));
 }
 
+avits_status avits_score_spatial_keymask(const void* q_img, const void* k_all, avits_dtype dt,
+                                         int B, int H, int M, int Nk, int d, int64_t q_sb,
+                                         int64_t q_sh, int64_t q_sn, int64_t k_sb, int64_t k_sh,
+                                         int64_t k_sn, const uint8_t* text_mask,
+                                         float softmax_scale, float weight, int accumulate,
+                                         float* A, float* lse_opt, void* workspace,
+                                         size_t ws_bytes, void* stream) {
+  if (!q_img || !k_all || !A || !text_mask || !valid_dtype(dt)) return AVITS_ERR_INVALID_ARG;
+  if (B <= 0 || H <= 0 || M <= 0 || Nk <= 0 || d <= 0 || Nk < M) return AVITS_ERR_INVALID_ARG;
+  if (!(softmax_scale > 0.f) || !(softmax_scale < 3.0e38f)) return AVITS_ERR_INVALID_ARG;
+  if (q_sn < d || k_sn < d || q_sh < 0 || k_sh < 0 || q_sb < 0 || k_sb < 0)
+    return AVITS_ERR_INVALID_ARG;
+  SpatialArgs a{q_img, k_all, dt, B, H, M, Nk, 0, d, q_sb, q_sh, q_sn, k_sb, k_sh, k_sn,
+                softmax_scale, weight, accumulate ? 1 : 0, A, lse_opt, workspace, ws_bytes,
+                status_word(), text_mask};
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (spatial_tc_eligible(a)) {
+    const int sms = num_sms_current();
+    if (ws_bytes < spatial_tc_workspace(B, H, M, Nk, d, sms) || !workspace)
+      return AVITS_ERR_INVALID_ARG;
+    return cuda_status(launch_spatial_tc(a, sms, s));
+  }
+  if (d > 256) return AVITS_ERR_UNSUPPORTED;
+  return cuda_status(launch_spatial_simt(a, s));
+}
+
 avits_status avits_score_temporal(const void* h_t, const void* h_prev, avits_dtype dt, int B,
                                   int N, int D, float eps, float* V, void* stream) {
   if (!h_t || !h_prev || !V || !valid_dtype(dt)) return AVITS_ERR_INVALID_ARG;

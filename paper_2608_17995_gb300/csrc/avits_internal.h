@@ -27,6 +27,7 @@ struct SpatialArgs {
   void* ws;
   size_t ws_bytes;
   unsigned int* status;
+  const uint8_t* tmask = nullptr;   // [B,Nk], nonzero = text key; NULL: keys j < L
 };
 
 // tcgen05 / TMA path (bf16, d in {64,128}); returns false if the shape or

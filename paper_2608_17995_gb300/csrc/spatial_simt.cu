@@ -6,7 +6,9 @@
 // the head mean of Eq. 3 is a fixed-order sum.  Per head, the query row sits
 // in shared memory; lanes stride over the keys, each keeping a running
 // (max, sum over all keys, sum over text keys) in the log2 domain; the lanes
-// are merged with shuffles.  text mass = sum_txt / sum_all.
+// are merged with shuffles.  text mass = sum_txt / sum_all.  The text keys
+// are the first L, or those a caller's key mask marks (interleaved text and
+// image keys).
 #include "avits_common.cuh"
 #include "avits_internal.h"
 
@@ -27,7 +29,8 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32)
 spatial_simt_kernel(const T* __restrict__ q, const T* __restrict__ k, int B, int H, int M, int Nk,
                     int L, int d, int64_t q_sb, int64_t q_sh, int64_t q_sn, int64_t k_sb,
                     int64_t k_sh, int64_t k_sn, float c_log2, float weight, int accumulate,
-                    float* __restrict__ A, float* __restrict__ lse) {
+                    float* __restrict__ A, float* __restrict__ lse,
+                    const uint8_t* __restrict__ tmask) {
   __shared__ float qs[kWarpsPerCta][kMaxD];
   const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
   const int64_t row = (int64_t)blockIdx.x * kWarpsPerCta + wl;
@@ -54,7 +57,7 @@ spatial_simt_kernel(const T* __restrict__ q, const T* __restrict__ k, int B, int
       }
       const float e = fast_ex2(x - m);
       la += e;
-      if (j < L) lt += e;
+      if (tmask ? tmask[(int64_t)b * Nk + j] != 0 : j < L) lt += e;
     }
     // merge the lanes
     float mw = m;
@@ -93,12 +96,12 @@ cudaError_t launch_spatial_simt(const SpatialArgs& a, cudaStream_t s) {
     spatial_simt_kernel<__nv_bfloat16><<<grid, kWarpsPerCta * 32, 0, s>>>(
         static_cast<const __nv_bfloat16*>(a.q), static_cast<const __nv_bfloat16*>(a.k), a.B, a.H,
         a.M, a.Nk, a.L, a.d, a.q_sb, a.q_sh, a.q_sn, a.k_sb, a.k_sh, a.k_sn, c_log2, a.weight,
-        a.accumulate, a.A, a.lse);
+        a.accumulate, a.A, a.lse, a.tmask);
   else
     spatial_simt_kernel<float><<<grid, kWarpsPerCta * 32, 0, s>>>(
         static_cast<const float*>(a.q), static_cast<const float*>(a.k), a.B, a.H, a.M, a.Nk, a.L,
         a.d, a.q_sb, a.q_sh, a.q_sn, a.k_sb, a.k_sh, a.k_sn, c_log2, a.weight, a.accumulate, a.A,
-        a.lse);
+        a.lse, a.tmask);
   return cudaGetLastError();
 }
 

@@ -99,6 +99,7 @@ struct TcParams {
   float* lse;
   float* part;      // [B*n_qp][H][2*max_parts][256][3]
   unsigned int* status;
+  const uint8_t* tmask;   // [B,Nk] text-key mask, or NULL (text keys = the first L)
 };
 
 // ------------------------------------------------------------------ PTX ----
@@ -362,20 +363,77 @@ __device__ __forceinline__ void process_chunk(const uint32_t (&r)[16], int col0,
 }
 
 // Kinds of the 64 keys a softmax warp reduces per item.
-enum ItemKind { kItemImage = 0, kItemText = 1, kItemGeneral = 2 };
+enum ItemKind { kItemImage = 0, kItemText = 1, kItemGeneral = 2, kItemMasked = 3 };
 
-// The 64 columns [c0, c0 + 64) of one S buffer for this warp's 32 rows: four
-// 16-column tcgen05.ld, each overlapped with the reduction of the previous
-// chunk.  The S buffer is handed back (arrive on s_empty) as soon as all 64
-// columns are in registers, before the last chunk is reduced.
+// A chunk whose text keys are given by a mask (bit e = key col0 + e is a text
+// key), possibly with invalid keys beyond Nk: the mixed case of a caller's
+// key mask.  Same lazy running maximum as process_chunk_full; the text sum
+// takes the exponentials of the masked keys.
+__device__ __forceinline__ void process_chunk_masked(const uint32_t (&r)[16], int col0, int Nk,
+                                                     uint32_t m16, float c, RowStat& st) {
+  float v[16];
+#pragma unroll
+  for (int e = 0; e < 16; ++e) v[e] = __uint_as_float(r[e]);
+  if (col0 + 16 > Nk) {
+#pragma unroll
+    for (int e = 0; e < 16; ++e)
+      if (col0 + e >= Nk) v[e] = -INFINITY;
+  }
+  const float nm = -st.m;
+  float ev[16];
+  float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+  for (int e = 0; e < 16; e += 4) {
+    float x0, x1, x2, x3;
+    ffma2(v[e], v[e + 1], c, nm, x0, x1);
+    ffma2(v[e + 2], v[e + 3], c, nm, x2, x3);
+    ev[e] = ex2(x0); ev[e + 1] = ex2(x1); ev[e + 2] = ex2(x2); ev[e + 3] = ex2(x3);
+    fadd2(s0, s1, ev[e], ev[e + 1]);
+    fadd2(s2, s3, ev[e + 2], ev[e + 3]);
+  }
+  fadd2(s0, s1, s2, s3);
+  float cs = s0 + s1;
+  if (!(cs < 0x1p64f)) {
+    // first chunk of a row, a logit 64 log2-units above the running maximum,
+    // or a NaN: the exact chunk maximum, then the exponentials again
+    float cm = v[0];
+#pragma unroll
+    for (int e = 1; e < 16; ++e) cm = fmaxf(cm, v[e]);
+    const float mx = fmaxf(st.m, cm * c);
+    if (mx == -INFINITY) return;   // no valid key
+    const float corr = ex2(st.m - mx);
+    st.la *= corr;
+    st.lt *= corr;
+    st.m = mx;
+    cs = 0.f;
+#pragma unroll
+    for (int e = 0; e < 16; ++e) {
+      ev[e] = ex2(fmaf(v[e], c, -mx));
+      cs += ev[e];
+    }
+  }
+  float t0 = 0.f, t1 = 0.f;
+#pragma unroll
+  for (int e = 0; e < 16; e += 2) {
+    t0 += ((m16 >> e) & 1u) ? ev[e] : 0.f;
+    t1 += ((m16 >> (e + 1)) & 1u) ? ev[e + 1] : 0.f;
+  }
+  st.la += cs;
+  st.lt += t0 + t1;
+}
+
 template <int kKind>
 __device__ __forceinline__ void softmax_item(uint32_t tb, int c0, int Nk, int L, float c,
-                                             RowStat& st, uint64_t* s_empty, int lane) {
+                                             RowStat& st, uint64_t* s_empty, int lane,
+                                             uint32_t w0 = 0u, uint32_t w1 = 0u) {
   uint32_t ra[16], rb[16];
-  const int nch = (kKind == kItemGeneral) ? max(0, min(4, (Nk - c0 + 15) >> 4)) : 4;
+  const int nch = (kKind >= kItemGeneral) ? max(0, min(4, (Nk - c0 + 15) >> 4)) : 4;
   auto chunk = [&](const uint32_t(&r)[16], int k) {
     if (kKind == kItemGeneral) {
       if (k < nch) process_chunk<0>(r, c0 + 16 * k, Nk, L, c, st);
+    } else if (kKind == kItemMasked) {
+      const uint32_t m16 = ((k < 2 ? w0 : w1) >> (16 * (k & 1))) & 0xFFFFu;
+      if (k < nch) process_chunk_masked(r, c0 + 16 * k, Nk, m16, c, st);
     } else {
       process_chunk_full<kKind == kItemText>(r, c, st);
     }
@@ -415,7 +473,9 @@ __device__ __forceinline__ int pieces(int u, int n_kt, int per) {
   return ((u + 1) * n_kt - 1) / per - (u * n_kt) / per + 1;
 }
 
-template <int D>
+// kMask: the text keys come from the caller's key mask (p.tmask) instead of
+// being the first L; a separate instance keeps the plain kernel unchanged.
+template <int D, bool kMask>
 __global__ void __launch_bounds__(kThreads, 1)
 spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                   const TcParams p) {
@@ -603,10 +663,19 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
     for (int it = it_begin; it < it_end;) {
       const Segment seg = segment_at(it, it_end, p.n_kt);
       RowStat st{-INFINITY, 0.f, 0.f};
+      const uint8_t* mrow = kMask ? p.tmask + (long long)((seg.u / p.n_qp) / p.H) * p.Nk : nullptr;
       for (int j = 0; j < seg.nk; ++j) {
         const int li = li0 + j;
         const int sb = li & 1;
         const uint32_t sph = (uint32_t)((li >> 1) & 1);
+        // the key mask does not depend on S: its bytes (lane l: keys c0 + l
+        // and c0 + 32 + l) are loaded before the wait for the S buffer
+        bool mb0 = false, mb1 = false;
+        if constexpr (kMask) {
+          const int cm0 = (seg.kt0 + j) * kBN + half * 64 + lane;
+          mb0 = cm0 < p.Nk && mrow[cm0] != 0;
+          mb1 = cm0 + 32 < p.Nk && mrow[cm0 + 32] != 0;
+        }
         bool ok = (*abort_flag == 0) && mbar_wait_bounded(&bars->s_full[t][sb], sph, abort_flag, p.status);
         ok = __all_sync(0xffffffffu, ok);   // tcgen05.ld below is warp-collective
         if (ok) {
@@ -615,7 +684,18 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
           const int c0 = (seg.kt0 + j) * kBN + half * 64;   // first key of this half
           uint64_t* empty = &bars->s_empty[t][sb];
           // the kind is uniform over the warp: one branch per item
-          if (c0 + 64 <= p.Nk && c0 + 64 <= p.L)
+          if constexpr (kMask) {
+            // the caller's key mask: bit l of w0 / w1 = key c0 + l / c0 + 32 + l
+            const uint32_t w0 = __ballot_sync(0xffffffffu, mb0);
+            const uint32_t w1 = __ballot_sync(0xffffffffu, mb1);
+            const bool full = c0 + 64 <= p.Nk;
+            if (full && (w0 & w1) == 0xffffffffu)
+              softmax_item<kItemText>(tb, c0, p.Nk, p.L, p.c_log2, st, empty, lane);
+            else if (full && (w0 | w1) == 0u)
+              softmax_item<kItemImage>(tb, c0, p.Nk, p.L, p.c_log2, st, empty, lane);
+            else
+              softmax_item<kItemMasked>(tb, c0, p.Nk, p.L, p.c_log2, st, empty, lane, w0, w1);
+          } else if (c0 + 64 <= p.Nk && c0 + 64 <= p.L)
             softmax_item<kItemText>(tb, c0, p.Nk, p.L, p.c_log2, st, empty, lane);
           else if (c0 + 64 <= p.Nk && c0 >= p.L)
             softmax_item<kItemImage>(tb, c0, p.Nk, p.L, p.c_log2, st, empty, lane);
@@ -782,6 +862,16 @@ bool strides_ok(int B, int H, int64_t sb, int64_t sh, int64_t sn) {
   return true;
 }
 
+// All-shared carveout and the dynamic shared-memory opt-in of one instance.
+template <auto Kernel, int D>
+cudaError_t smem_attrs() {
+  cudaError_t e = cudaFuncSetAttribute(Kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                       cudaSharedmemCarveoutMaxShared);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(Kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<D>());
+  return e;
+}
+
 // The dynamic shared-memory opt-in is a per-device function attribute: set it
 // once per device (first call, outside any stream capture in practice).
 cudaError_t set_smem_once() {
@@ -792,20 +882,13 @@ cudaError_t set_smem_once() {
   if (dev >= 0 && dev < 64 && __atomic_load_n(&done[dev], __ATOMIC_ACQUIRE)) return cudaSuccess;
   // one carveout (all shared) for every kernel of the path, so that kernels
   // launched as programmatic dependents can share an SM with this one
-  e = cudaFuncSetAttribute(spatial_tc_kernel<128>, cudaFuncAttributePreferredSharedMemoryCarveout,
-                           cudaSharedmemCarveoutMaxShared);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(spatial_tc_kernel<64>, cudaFuncAttributePreferredSharedMemoryCarveout,
-                             cudaSharedmemCarveoutMaxShared);
+  e = smem_attrs<spatial_tc_kernel<128, false>, 128>();
+  if (e == cudaSuccess) e = smem_attrs<spatial_tc_kernel<128, true>, 128>();
+  if (e == cudaSuccess) e = smem_attrs<spatial_tc_kernel<64, false>, 64>();
+  if (e == cudaSuccess) e = smem_attrs<spatial_tc_kernel<64, true>, 64>();
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(spatial_finalize_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
                              cudaSharedmemCarveoutMaxShared);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(spatial_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             smem_bytes<128>());
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(spatial_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             smem_bytes<64>());
   if (e == cudaSuccess && dev >= 0 && dev < 64) __atomic_store_n(&done[dev], 1, __ATOMIC_RELEASE);
   return e;
 }
@@ -848,14 +931,16 @@ cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s,
   p.lse = a.lse;
   p.part = reinterpret_cast<float*>(ws);
   p.status = a.status;
+  p.tmask = a.tmask;
   cudaError_t e = set_smem_once();
   if (e != cudaSuccess) return e;
+  const bool masked = p.tmask != nullptr;
   if (a.d == 128)
-    e = launch_pdl(spatial_tc_kernel<128>, dim3(pl.grid), dim3(kThreads), smem_bytes<128>(), s, mq,
-                   mk, p);
+    e = launch_pdl(masked ? spatial_tc_kernel<128, true> : spatial_tc_kernel<128, false>,
+                   dim3(pl.grid), dim3(kThreads), smem_bytes<128>(), s, mq, mk, p);
   else
-    e = launch_pdl(spatial_tc_kernel<64>, dim3(pl.grid), dim3(kThreads), smem_bytes<64>(), s, mq,
-                   mk, p);
+    e = launch_pdl(masked ? spatial_tc_kernel<64, true> : spatial_tc_kernel<64, false>,
+                   dim3(pl.grid), dim3(kThreads), smem_bytes<64>(), s, mq, mk, p);
   if (e != cudaSuccess) return e;
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;

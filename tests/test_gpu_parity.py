@@ -85,6 +85,86 @@ def _check_spatial(av, orc, q, k, L, scale, dtype, rows=None, rtol=BF16_RTOL, we
     return A_g
 
 
+def _check_spatial_mask(av, orc, q, k, mask, scale, dtype, rows=None, rtol=BF16_RTOL):
+    """avits_score_spatial_keymask against the masked oracle (A and the
+    per-head mass through the lse pair)."""
+    import torch
+    B, H, M, d = q.shape
+    A = torch.zeros(B, M, dtype=torch.float32, device="cuda")
+    lse = torch.zeros(B, H, M, 2, dtype=torch.float32, device="cuda")
+    md = torch.from_numpy(np.ascontiguousarray(mask.astype(np.uint8))).cuda()
+    av.avits_score_spatial(_dev(q, dtype), _dev(k, dtype), 0, scale, A, lse=lse, text_mask=md)
+    assert _status(av) == 0
+    A_o, mass_o, _ = orc.score_spatial(q, k, 0, scale, rows=rows, text_mask=mask)
+    A_g, lse_g = _np(A), _np(lse)
+    idx = np.arange(B * M) if rows is None else np.asarray(rows)
+    np.testing.assert_allclose(A_g.ravel()[idx], A_o.ravel()[idx], rtol=rtol, atol=1e-6)
+    b_i = np.stack([idx // M, idx % M], 1)
+    for h in range(H):
+        mg = np.exp(lse_g[b_i[:, 0], h, b_i[:, 1], 1] - lse_g[b_i[:, 0], h, b_i[:, 1], 0])
+        np.testing.assert_allclose(mg, mass_o[b_i[:, 0], h, b_i[:, 1]],
+                                   rtol=max(rtol, 1e-5) * 2, atol=1e-6)
+    return A_g
+
+
+def test_spatial_keymask_fp32(av, orc):
+    """Interleaved text keys, CUDA-core path (fp32)."""
+    from paper_2608_17995_gb300.workloads import make_transition
+    tr = make_transition("tiny")
+    rng = np.random.default_rng(3)
+    mask = (rng.random((tr.B, tr.Nk)) < 0.2).astype(np.uint8)
+    _check_spatial_mask(av, orc, tr.q_img, tr.k_all, mask, tr.softmax_scale, "f32", rtol=F32_TOL)
+
+
+@pytest.mark.parametrize("B,H,M,Nk,d,kind", [(1, 24, 1024, 1536, 128, "random"),
+                                             (2, 4, 300, 1333, 128, "blocks"),
+                                             (1, 6, 256, 700, 64, "random"),
+                                             (1, 8, 512, 1024, 128, "none"),
+                                             (1, 8, 512, 1024, 128, "all")])
+def test_spatial_keymask_bf16(av, orc, B, H, M, Nk, d, kind):
+    """Interleaved text keys on the tensor-core path: random masks (every
+    item mixed), text blocks at arbitrary offsets (full text, full image and
+    mixed items), ragged key counts, d = 64, and the empty / full masks."""
+    from paper_2608_17995_gb300.workloads import to_bf16_bits
+    rng = np.random.default_rng(M + Nk)
+    q = to_bf16_bits((rng.standard_normal((B, H, M, d)) * 0.3).astype(np.float32))
+    k = to_bf16_bits((rng.standard_normal((B, H, Nk, d)) * 0.3).astype(np.float32))
+    if kind == "random":
+        mask = (rng.random((B, Nk)) < 0.3).astype(np.uint8)
+    elif kind == "blocks":
+        mask = np.zeros((B, Nk), np.uint8)
+        mask[:, 77:301] = 1
+        mask[:, 640:768] = 1          # one whole 128-key tile
+        mask[:, 1290:1333] = 1        # up to the ragged end
+    elif kind == "none":
+        mask = np.zeros((B, Nk), np.uint8)
+    else:
+        mask = np.ones((B, Nk), np.uint8)
+    rows = _sample_rows(B, M, 64, seed=5)
+    A = _check_spatial_mask(av, orc, q, k, mask, 1.0 / math.sqrt(d), "bf16", rows=rows)
+    if kind == "none":
+        assert np.all(A == 0.0)
+    if kind == "all":
+        np.testing.assert_allclose(A, 1.0, rtol=1e-6)
+
+
+def test_spatial_keymask_first_l_is_l_form(av, orc):
+    """A mask of the first 512 keys (a multiple of the 64-key halves) takes
+    the same item paths as the L form: bit-identical A at the FLUX-1024 shape."""
+    import torch
+    from paper_2608_17995_gb300.workloads import make_transition
+    tr = make_transition("flux1024")
+    q, k = _dev(tr.q_img, "bf16"), _dev(tr.k_all, "bf16")
+    A1 = torch.zeros(tr.B, tr.M, dtype=torch.float32, device="cuda")
+    A2 = torch.zeros_like(A1)
+    av.avits_score_spatial(q, k, tr.L, tr.softmax_scale, A1)
+    mask = torch.zeros(tr.B, tr.Nk, dtype=torch.uint8, device="cuda")
+    mask[:, :tr.L] = 1
+    av.avits_score_spatial(q, k, 0, tr.softmax_scale, A2, text_mask=mask)
+    assert _status(av) == 0
+    assert torch.equal(A1.view(torch.int32), A2.view(torch.int32))
+
+
 def test_spatial_tiny_fp32(av, orc):
     from paper_2608_17995_gb300.workloads import make_transition
     tr = make_transition("tiny")
