@@ -160,6 +160,9 @@ def algorithmic_work(tr, mode):
         "temporal": {"bytes": float(2 * B * M * D * elt + 4 * B * M)},
         "select": {"bytes": float(8 * B * M + 4 * B * M + 4 * B * tr.k + B * M + 4 * B * M)},
         "upsample": {"bytes": float(B * M * T * elt + B * M * 5 + B * NO * (T * elt + 17))},
+        "select_upsample": {"bytes": float(8 * B * M + 4 * B * M + 4 * B * tr.k + B * M
+                                           + 4 * B * M + B * M * T * elt
+                                           + B * NO * (T * elt + 17))},
         "merge": {"bytes": float(B * NO * (T * elt + 12) + B * F * T * elt)},
     }
 
@@ -228,9 +231,10 @@ def run_ours(args, world, rank, local, pg):
     sets = [base] + [tuple(t.clone() for t in base) for _ in range(nsets - 1)]
     torch.cuda.synchronize()
 
-    # spatial = scores + merge kernel; bilinear merge = map + gather kernels
-    kernels_per_step = 6 if buf.mode == av.NEAREST else 7
-    names = ["spatial", "temporal", "select", "upsample", "merge"]
+    # our kernels per step: spatial main + temporal (beside it) + finalize,
+    # the fused selection + upsample, the merge (bilinear: map + gather)
+    kernels_per_step = 5 if buf.mode == av.NEAREST else 6
+    names = ["spatial", "temporal", "select", "upsample", "merge", "select_upsample"]
 
     def step(s, st):
         buf.set_inputs(*sets[s % nsets])
@@ -371,7 +375,8 @@ def per_kernel_times(torch, av, buf, sets, nsets, stream, names, args):
     time includes its in-graph launch gap; avits_score_spatial is two kernels
     (scores + merge)."""
     calls = {"spatial": buf.spatial, "temporal": buf.temporal, "select": buf.select,
-             "upsample": buf.upsample, "merge": buf.merge}
+             "upsample": buf.upsample, "merge": buf.merge,
+             "select_upsample": buf.select_upsample}
     n, reps = max(nsets * 4, 48), 10
     out = {"_how": "graph of %d back-to-back calls per entry point, %d replays" % (n, reps)}
     for name in names:

@@ -277,6 +277,27 @@ avits_status avits_selective_upsample(const void* latent, avits_dtype dt, int B,
                                       int8_t* out_src_sub, void* stream);
 
 /* ------------------------------------------------------------------------
+ * avits_fuse_select_perturbed followed by avits_selective_upsample, in ONE
+ * launch (the transition of Sec. 3.2 after Eq. 8-9): every output is what
+ * the two calls produce, bit for bit.  Each batch element gets several CTAs
+ * that all compute its selection, so none waits for another; the first one
+ * writes S_opt, sel_idx, sel_mask and tok_offset.  Up to M = 2048 tokens per
+ * element it is one kernel; above that the two kernels run back to back.
+ * perturb : NULL or [B,M] fp32 (Eq. 9 tie-breaking noise, as
+ *           avits_fuse_select_perturbed).
+ * sel_mask : REQUIRED here ([B,M] uint8).  The remaining arguments are those
+ *            of avits_fuse_select_perturbed and avits_selective_upsample.
+ * ---------------------------------------------------------------------- */
+avits_status avits_select_upsample(const float* A, const float* V, const float* perturb, int B,
+                                   int M, float alpha, float eps_norm, int k, float* S_opt,
+                                   int32_t* sel_idx, uint8_t* sel_mask, int32_t* tok_offset,
+                                   const void* latent, avits_dtype dt, int grid_h, int grid_w,
+                                   int C, int p, const int32_t* pos_in_opt,
+                                   const int32_t* span_in_opt, avits_upmode mode,
+                                   void* out_latent, int32_t* out_pos, int32_t* out_span,
+                                   int32_t* out_src_tok, int8_t* out_src_sub, void* stream);
+
+/* ------------------------------------------------------------------------
  * Final merge, Sec. 3.2 Stage 3: expand every remaining token to full
  * resolution and lay the tokens out in spatial (raster) order.
  * A token at (y,x) with span s covers cells [y,y+s) x [x,x+s) of the

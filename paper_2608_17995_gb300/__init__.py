@@ -81,6 +81,8 @@ def lib():
         "avits_fuse_select_perturbed": [vp, vp, vp, i32, i32, f32, f32, i32, vp, vp, vp, vp, vp],
         "avits_selective_upsample": [vp, i32, i32, i32, i32, i32, i32, i32, vp, vp, vp, vp, i32,
                                      i32, vp, vp, vp, vp, vp, vp],
+        "avits_select_upsample": [vp, vp, vp, i32, i32, f32, f32, i32, vp, vp, vp, vp, vp, i32,
+                                  i32, i32, i32, i32, vp, vp, i32, vp, vp, vp, vp, vp, vp],
         "avits_merge_final": [vp, i32, i32, i32, vp, vp, i32, i32, i32, i32, i32, vp, vp, sz, vp],
         "avits_merge_final_workspace": [i32, i32, i32, i32],
         "avits_device_status": [vp],
@@ -292,6 +294,23 @@ def avits_fuse_select(A, V, alpha: float, k: int, sel_idx, tok_offset, S=None, s
                                                _ptr(sel_idx), _ptr(sel_mask), _ptr(tok_offset),
                                                _stream(stream))
         _check("avits_fuse_select_perturbed", rc)
+    return sel_idx
+
+
+def avits_select_upsample(A, V, alpha: float, k: int, sel_idx, tok_offset, sel_mask, latent,
+                          grid_h: int, grid_w: int, out_latent, out_pos, out_span, out_src_tok,
+                          out_src_sub, S=None, perturb=None, mode: int = NEAREST, pos_in=None,
+                          span_in=None, eps_norm: float = 1e-6, stream=None):
+    """avits_fuse_select(_perturbed) + avits_selective_upsample in one launch;
+    the same outputs as the two calls."""
+    B, M = A.shape
+    T = latent.shape[2]
+    rc = lib().avits_select_upsample(
+        _ptr(A), _ptr(V), _ptr(perturb), B, M, float(alpha), float(eps_norm), int(k), _ptr(S),
+        _ptr(sel_idx), _ptr(sel_mask), _ptr(tok_offset), _ptr(latent), _dtype_code(latent),
+        grid_h, grid_w, T // 4, 2, _ptr(pos_in), _ptr(span_in), int(mode), _ptr(out_latent),
+        _ptr(out_pos), _ptr(out_span), _ptr(out_src_tok), _ptr(out_src_sub), _stream(stream))
+    _check("avits_select_upsample", rc)
     return sel_idx
 
 

@@ -232,6 +232,33 @@ avits_status avits_selective_upsample(const void* latent, avits_dtype dt, int B,
                                      static_cast<cudaStream_t>(stream)));
 }
 
+avits_status avits_select_upsample(const float* A, const float* V, const float* perturb, int B,
+                                   int M, float alpha, float eps_norm, int k, float* S_opt,
+                                   int32_t* sel_idx, uint8_t* sel_mask, int32_t* tok_offset,
+                                   const void* latent, avits_dtype dt, int grid_h, int grid_w,
+                                   int C, int p, const int32_t* pos_in_opt,
+                                   const int32_t* span_in_opt, avits_upmode mode,
+                                   void* out_latent, int32_t* out_pos, int32_t* out_span,
+                                   int32_t* out_src_tok, int8_t* out_src_sub, void* stream) {
+  if (!A || !V || !tok_offset || !sel_mask || (k > 0 && !sel_idx)) return AVITS_ERR_INVALID_ARG;
+  if (B <= 0 || M <= 0 || M > kSelectMaxM || k < 0 || k > M) return AVITS_ERR_INVALID_ARG;
+  if (!(alpha >= 0.f && alpha <= 1.f) || !(eps_norm >= 0.f)) return AVITS_ERR_INVALID_ARG;
+  if (!latent || !out_latent || !out_pos || !out_span || !out_src_tok || !out_src_sub ||
+      !valid_dtype(dt))
+    return AVITS_ERR_INVALID_ARG;
+  if (grid_h <= 0 || grid_w <= 0 || C <= 0) return AVITS_ERR_INVALID_ARG;
+  if (p != 2) return AVITS_ERR_UNSUPPORTED;
+  if ((pos_in_opt == nullptr) != (span_in_opt == nullptr)) return AVITS_ERR_INVALID_ARG;
+  if (!pos_in_opt && (int64_t)grid_h * grid_w != M) return AVITS_ERR_INVALID_ARG;
+  if (mode != AVITS_UP_NEAREST && mode != AVITS_UP_BILINEAR) return AVITS_ERR_INVALID_ARG;
+  if (mode == AVITS_UP_BILINEAR && pos_in_opt) return AVITS_ERR_UNSUPPORTED;
+  if (!aligned16(latent) || !aligned16(out_latent)) return AVITS_ERR_INVALID_ARG;
+  return cuda_status(launch_select_upsample(
+      A, V, perturb, B, M, alpha, eps_norm, k, S_opt, sel_idx, sel_mask, tok_offset,
+      status_word(), latent, dt, grid_h, grid_w, C, pos_in_opt, span_in_opt, mode, out_latent,
+      out_pos, out_span, out_src_tok, out_src_sub, static_cast<cudaStream_t>(stream)));
+}
+
 size_t avits_merge_final_workspace(avits_upmode mode, int B, int full_h, int full_w) {
   if (mode != AVITS_UP_BILINEAR || B <= 0 || full_h <= 0 || full_w <= 0) return 0;
   return sizeof(int32_t) * (size_t)B * full_h * full_w;

@@ -62,6 +62,15 @@ cudaError_t launch_fuse_select(const float* A, const float* V, const float* pert
                                cudaStream_t s);
 
 // ---- selective upsample (Stage 2) -------------------------------------------
+// Selection + selective upsample in one launch (two above 2048 tokens).
+cudaError_t launch_select_upsample(const float* A, const float* V, const float* perturb, int B,
+                                   int M, float alpha, float eps, int k, float* S,
+                                   int32_t* sel_idx, uint8_t* mask, int32_t* tok_offset,
+                                   unsigned int* status, const void* latent, avits_dtype dt,
+                                   int gh, int gw, int C, const int32_t* pos_in,
+                                   const int32_t* span_in, avits_upmode mode, void* out,
+                                   int32_t* out_pos, int32_t* out_span, int32_t* out_src_tok,
+                                   int8_t* out_src_sub, cudaStream_t s);
 cudaError_t launch_upsample(const void* latent, avits_dtype dt, int B, int M, int gh, int gw,
                             int C, const int32_t* pos_in, const int32_t* span_in,
                             const uint8_t* mask, const int32_t* tok_offset, int k,

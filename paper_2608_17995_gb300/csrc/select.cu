@@ -26,6 +26,7 @@
 //      it yields sel_idx (ascending), the mask and tok_offset.
 #include "avits_common.cuh"
 #include "avits_internal.h"
+#include "upsample_token.cuh"
 
 namespace avits {
 namespace {
@@ -58,24 +59,45 @@ __device__ __forceinline__ uint32_t count_digits(uint32_t key, bool valid, uint3
   return __popc(m);
 }
 
-// kRegKeys keys per thread in registers when M <= kRegKeys * kThreads; larger
-// M (kRegKeys = 0) keeps them in shared memory only.
+struct SelArgs {
+  const float* A;
+  const float* V;
+  const float* perturb;   // NULL or [B,M]
+  int M;
+  float alpha, eps;
+  int k;
+  float* S_out;           // NULL or [B,M]
+  int32_t* sel_idx;
+  uint8_t* mask;          // NULL or [B,M]
+  int32_t* tok_offset;
+  unsigned int* status;
+};
+
+// The selection of batch element b by one CTA.  kRegKeys keys per thread in
+// registers when M <= kRegKeys * kThreads; larger M (kRegKeys = 0) keeps them
+// in shared memory only.  `keys` is the CTA's dynamic shared memory (M words).
+// write_out: this CTA writes S, sel_idx, the mask and tok_offset.  offs_s /
+// sel_s (or NULL): every token's start in the mixed sequence and whether it
+// is selected, left in shared memory for the fused upsample.
 template <int kThreads, int kRegKeys>
-__global__ void __launch_bounds__(kThreads)
-fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V,
-                   const float* __restrict__ perturb, int M, float alpha,
-                   float eps, int k, float* __restrict__ S_out, int32_t* __restrict__ sel_idx,
-                   uint8_t* __restrict__ mask, int32_t* __restrict__ tok_offset,
-                   unsigned int* status) {
+__device__ __forceinline__ void select_body(const SelArgs& g, int b, bool write_out,
+                                            uint32_t* keys, int32_t* offs_s, uint8_t* sel_s) {
   constexpr int kWarps = kThreads / 32;
-  extern __shared__ uint32_t keys[];
   __shared__ float red[4][kWarps];
   __shared__ uint32_t cnt[2][kWarps][16];
   __shared__ uint32_t scan_tot[kWarps];
   __shared__ int sh_nan;
+  const float* __restrict__ A = g.A;
+  const float* __restrict__ V = g.V;
+  const float* __restrict__ perturb = g.perturb;
+  const int M = g.M, k = g.k;
+  const float alpha = g.alpha, eps = g.eps;
+  float* __restrict__ S_out = write_out ? g.S_out : nullptr;
+  int32_t* __restrict__ sel_idx = g.sel_idx;
+  uint8_t* __restrict__ mask = g.mask;
+  int32_t* __restrict__ tok_offset = g.tok_offset;
 
   pdl_wait_then_trigger();
-  const int b = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   const float* a = A + (int64_t)b * M;
   const float* v = V + (int64_t)b * M;
@@ -220,7 +242,7 @@ fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V,
   // is above T are in; of the keys with prefix T the `remaining` lowest indices
   const uint32_t T = shift < 32 ? (prefix >> shift) : 0u;
   __syncthreads();   // keys[] complete for the range pass below
-  if (tid == 0 && sh_nan) raise_status(status, AVITS_ERR_NAN);
+  if (write_out && tid == 0 && sh_nan) raise_status(g.status, AVITS_ERR_NAN);
 
   // 4. one scan of (above, equal) over contiguous per-thread ranges
   const int per = (M + kThreads - 1) / kThreads;
@@ -262,9 +284,75 @@ fuse_select_kernel(const float* __restrict__ A, const float* __restrict__ V,
       sel = kp > T;
       if (kp == T) { sel = eq_seen < remaining; ++eq_seen; }
     }
-    tok_offset[(int64_t)b * M + i] = i + 3 * (int)c;
-    if (mask) mask[(int64_t)b * M + i] = sel ? 1 : 0;
-    if (sel) { sel_idx[(int64_t)b * k + c] = i; ++c; }
+    if (write_out) {
+      tok_offset[(int64_t)b * M + i] = i + 3 * (int)c;
+      if (mask) mask[(int64_t)b * M + i] = sel ? 1 : 0;
+      if (sel) sel_idx[(int64_t)b * k + c] = i;
+    }
+    if (offs_s) {
+      offs_s[i] = i + 3 * (int)c;
+      sel_s[i] = sel ? 1 : 0;
+    }
+    if (sel) ++c;
+  }
+}
+
+template <int kThreads, int kRegKeys>
+__global__ void __launch_bounds__(kThreads)
+fuse_select_kernel(const SelArgs g) {
+  extern __shared__ uint32_t keys[];
+  select_body<kThreads, kRegKeys>(g, blockIdx.x, true, keys, nullptr, nullptr);
+}
+
+// One-launch selection + selective upsample (Eq. 8-9, then Sec. 3.2 Stage
+// 2).  The grid has `parts` CTAs per batch element, CTA `part` owning the
+// contiguous tokens [lo, hi).  Every CTA first starts copying the latent
+// rows it will read (its tokens, and for bilinear the neighbouring grid rows)
+// into shared memory with cp.async, then computes the element's selection
+// (latency-bound work, so the redundant copies only occupy otherwise idle
+// SMs) while the copy lands; part 0 writes the selection outputs; finally
+// each warp upsamples its tokens from shared memory.  No CTA waits for
+// another.
+template <int kThreads, int kRegKeys, typename T, bool kBilinear>
+__global__ void __launch_bounds__(kThreads)
+select_upsample_kernel(const SelArgs g, const UpsampleArgs<T> u, int parts, int stage_rows) {
+  extern __shared__ uint32_t keys[];
+  const int b = blockIdx.x / parts, part = blockIdx.x - b * parts;
+  const int M = g.M, T4 = u.C * 4;
+  int32_t* offs_s = reinterpret_cast<int32_t*>(keys + M);
+  uint8_t* sel_s = reinterpret_cast<uint8_t*>(offs_s + M);
+  T* rows_s = reinterpret_cast<T*>(keys + ((9 * M + 15) / 16) * 4);   // 16-byte aligned
+  const int chunk = (M + parts - 1) / parts;
+  const int lo = min(M, part * chunk), hi = min(M, lo + chunk);
+  const int halo = kBilinear ? u.gw + 1 : 0;
+  const int s_lo = max(0, lo - halo), s_hi = min(M, hi + halo);
+  // the latent is an input of this kernel: read it after the wait on the
+  // kernel before (select_body's first step), so issue the copy just after
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const bool staged = stage_rows > 0;
+  if (staged) {
+    const char* src = reinterpret_cast<const char*>(u.latent + ((int64_t)b * M + s_lo) * T4);
+    char* dst = reinterpret_cast<char*>(rows_s);
+    const int n16 = (s_hi - s_lo) * T4 * (int)sizeof(T) / 16;
+    for (int q = threadIdx.x; q < n16; q += kThreads)
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst + 16 * q)),
+                   "l"(src + 16 * q)
+                   : "memory");
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  }
+  select_body<kThreads, kRegKeys>(g, b, part == 0, keys, offs_s, sel_s);
+  if (staged) asm volatile("cp.async.wait_all;" ::: "memory");
+  __syncthreads();
+  constexpr int kWarps = kThreads / 32;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  if (staged) {
+    const SharedRows<T> rows{rows_s, s_lo, T4};
+    for (int i = lo + w; i < hi; i += kWarps)
+      upsample_token<T, kBilinear>(u, rows, b, i, offs_s[i], sel_s[i] != 0, lane);
+  } else {
+    const GlobalRows<T> rows{u.latent, M, T4};
+    for (int i = lo + w; i < hi; i += kWarps)
+      upsample_token<T, kBilinear>(u, rows, b, i, offs_s[i], sel_s[i] != 0, lane);
   }
 }
 
@@ -294,8 +382,7 @@ cudaError_t launch_fuse_select(const float* A, const float* V, const float* pert
   }
   // 256 threads up to M = 1024 (fewer warps to synchronise and scan over,
   // measured faster at FLUX-1024), 512 beyond; shared memory only above 4096
-  void (*kern)(const float*, const float*, const float*, int, float, float, int, float*,
-               int32_t*, uint8_t*, int32_t*, unsigned int*);
+  void (*kern)(const SelArgs);
   int threads;
   if (M <= 1024) {
     threads = 256;
@@ -317,10 +404,91 @@ cudaError_t launch_fuse_select(const float* A, const float* V, const float* pert
   if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<kMaxThreads, kMaxRegKeys>>();
   if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<kMaxThreads, 0>>();
   if (ce != cudaSuccess) return ce;
-  cudaError_t e = launch_pdl(kern, dim3(B), dim3(threads), smem, s, A, V, perturb, M, alpha, eps,
-                             k, S, sel_idx, mask, tok_offset, status);
+  const SelArgs g{A, V, perturb, M, alpha, eps, k, S, sel_idx, mask, tok_offset, status};
+  cudaError_t e = launch_pdl(kern, dim3(B), dim3(threads), smem, s, g);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
+}
+
+namespace {
+
+constexpr int kFusedThreads = 256;
+constexpr int kFusedCtasTotal = 152;   // CTAs of the fused kernel over all elements
+constexpr int kFusedMaxM = kFusedThreads * kMaxRegKeys;   // 2048
+
+template <typename T, bool kBilinear>
+cudaError_t launch_fused_t(const SelArgs& g, const UpsampleArgs<T>& u, int B, int M,
+                           cudaStream_t s) {
+  const int per = (M + kFusedThreads - 1) / kFusedThreads;
+  auto kern = per <= 1   ? select_upsample_kernel<kFusedThreads, 1, T, kBilinear>
+              : per <= 2 ? select_upsample_kernel<kFusedThreads, 2, T, kBilinear>
+              : per <= 4 ? select_upsample_kernel<kFusedThreads, 4, T, kBilinear>
+                         : select_upsample_kernel<kFusedThreads, 8, T, kBilinear>;
+  cudaError_t e = prefer_max_shared<select_upsample_kernel<kFusedThreads, 1, T, kBilinear>>();
+  if (e == cudaSuccess) e = prefer_max_shared<select_upsample_kernel<kFusedThreads, 2, T, kBilinear>>();
+  if (e == cudaSuccess) e = prefer_max_shared<select_upsample_kernel<kFusedThreads, 4, T, kBilinear>>();
+  if (e == cudaSuccess) e = prefer_max_shared<select_upsample_kernel<kFusedThreads, 8, T, kBilinear>>();
+  if (e != cudaSuccess) return e;
+  // about 2 tokens per warp, at most one CTA per SM over all elements (every
+  // CTA repeats its element's selection)
+  const int parts = std::max(1, std::min((M + 15) / 16, std::max(1, kFusedCtasTotal / B)));
+  const int chunk = (M + parts - 1) / parts;
+  const int halo = kBilinear ? u.gw + 1 : 0;
+  const size_t row_bytes = (size_t)u.C * 4 * sizeof(T);
+  // rows copied to shared memory: the CTA's tokens and their bilinear
+  // neighbours, when rows are whole 16-byte copies and the copy fits
+  int stage_rows = std::min(M, chunk + 2 * halo);
+  const size_t head = ((9 * (size_t)M + 15) / 16) * 16;
+  if (row_bytes % 16 != 0 || (reinterpret_cast<uintptr_t>(u.latent) & 15u) != 0 ||
+      head + stage_rows * row_bytes > 96 * 1024)
+    stage_rows = 0;
+  const size_t smem = head + (size_t)stage_rows * row_bytes;
+  if (smem > 48 * 1024) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
+    if (e != cudaSuccess) return e;
+  }
+  e = launch_pdl(kern, dim3((unsigned)(B * parts)), dim3(kFusedThreads), smem, s, g, u, parts,
+                 stage_rows);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t launch_fused_mode(const SelArgs& g, const void* latent, int B, int M, int gh, int gw,
+                              int C, const int32_t* pos_in, const int32_t* span_in,
+                              avits_upmode mode, void* out, int32_t* out_pos, int32_t* out_span,
+                              int32_t* out_src_tok, int8_t* out_src_sub, cudaStream_t s) {
+  const UpsampleArgs<T> u{static_cast<const T*>(latent), M, gh, gw, C, M + 3 * g.k, pos_in,
+                          span_in, static_cast<T*>(out), out_pos, out_span, out_src_tok,
+                          out_src_sub};
+  return mode == AVITS_UP_BILINEAR ? launch_fused_t<T, true>(g, u, B, M, s)
+                                   : launch_fused_t<T, false>(g, u, B, M, s);
+}
+
+}  // namespace
+
+cudaError_t launch_select_upsample(const float* A, const float* V, const float* perturb, int B,
+                                   int M, float alpha, float eps, int k, float* S,
+                                   int32_t* sel_idx, uint8_t* mask, int32_t* tok_offset,
+                                   unsigned int* status, const void* latent, avits_dtype dt,
+                                   int gh, int gw, int C, const int32_t* pos_in,
+                                   const int32_t* span_in, avits_upmode mode, void* out,
+                                   int32_t* out_pos, int32_t* out_span, int32_t* out_src_tok,
+                                   int8_t* out_src_sub, cudaStream_t s) {
+  if (M > kFusedMaxM) {
+    // beyond one CTA's registers: the two launches, same outputs
+    cudaError_t e = launch_fuse_select(A, V, perturb, B, M, alpha, eps, k, S, sel_idx, mask,
+                                       tok_offset, status, s);
+    if (e != cudaSuccess) return e;
+    return launch_upsample(latent, dt, B, M, gh, gw, C, pos_in, span_in, mask, tok_offset, k,
+                           mode, out, out_pos, out_span, out_src_tok, out_src_sub, s);
+  }
+  const SelArgs g{A, V, perturb, M, alpha, eps, k, S, sel_idx, mask, tok_offset, status};
+  if (dt == AVITS_BF16)
+    return launch_fused_mode<__nv_bfloat16>(g, latent, B, M, gh, gw, C, pos_in, span_in, mode,
+                                             out, out_pos, out_span, out_src_tok, out_src_sub, s);
+  return launch_fused_mode<float>(g, latent, B, M, gh, gw, C, pos_in, span_in, mode, out, out_pos,
+                                  out_span, out_src_tok, out_src_sub, s);
 }
 
 }  // namespace avits

@@ -2,8 +2,8 @@
 
 Plumbing only: it owns the output tensors and the workspaces and issues
 avits_score_spatiotemporal (or avits_score_spatial + avits_score_temporal) ->
-avits_fuse_select -> avits_selective_upsample -> avits_merge_final on one
-stream.
+avits_select_upsample (or avits_fuse_select + avits_selective_upsample) ->
+avits_merge_final on one stream.
 """
 from __future__ import annotations
 
@@ -11,7 +11,7 @@ import numpy as np
 
 from . import (BILINEAR, NEAREST, SpatialWorkspace, avits_fuse_select, avits_merge_final,
                avits_merge_final_workspace, avits_score_spatial, avits_score_spatiotemporal,
-               avits_score_temporal, avits_selective_upsample)
+               avits_score_temporal, avits_select_upsample, avits_selective_upsample)
 
 
 def to_device(arr: np.ndarray, dtype: str, device="cuda"):
@@ -98,14 +98,23 @@ class TransitionBuffers:
                                  self.src_tok, self.src_sub, mode=self.mode, pos_in=self.pos_in,
                                  span_in=self.span_in, stream=stream)
 
+    def select_upsample(self, stream=None):
+        """Selection and selective upsampling in one launch."""
+        avits_select_upsample(self.A, self.V, self.tr.alpha, self.tr.k, self.sel_idx,
+                              self.tok_offset, self.sel_mask, self.latent, self.tr.frame_h,
+                              self.tr.frame_w, self.mixed, self.pos, self.span, self.src_tok,
+                              self.src_sub, S=self.S, mode=self.mode, pos_in=self.pos_in,
+                              span_in=self.span_in, stream=stream)
+
     def merge(self, stream=None):
         avits_merge_final(self.mixed, self.pos, self.span, self.full_h, self.full_w, self.full,
                           mode=self.mode, workspace=self.merge_ws, stream=stream)
 
-    def run(self, stream=None, merge=True, fused_scores=True):
+    def run(self, stream=None, merge=True, fused_scores=True, fused_tail=True):
         """The transition on one stream: both scores (one call, the temporal
         kernel overlapping the spatial one, unless fused_scores=False), then
-        selection, selective upsampling and the final merge."""
+        selection and selective upsampling (one launch unless
+        fused_tail=False) and the final merge."""
         import torch
         main = stream if stream is not None else torch.cuda.current_stream()
         if fused_scores:
@@ -113,7 +122,10 @@ class TransitionBuffers:
         else:
             self.spatial(main)
             self.temporal(main)
-        self.select(main)
-        self.upsample(main)
+        if fused_tail:
+            self.select_upsample(main)
+        else:
+            self.select(main)
+            self.upsample(main)
         if merge:
             self.merge(main)

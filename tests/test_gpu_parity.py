@@ -517,6 +517,83 @@ def test_transition_end_to_end(av, orc, name):
     assert np.array_equal(_bits(_np(buf.full)), _bits(full_o))
 
 
+def _fused_vs_separate(av, buf, perturb=None, k=None):
+    """avits_select_upsample against avits_fuse_select + avits_selective_upsample
+    on the same inputs: every output bit-identical."""
+    import torch
+    tr = buf.tr
+    k = tr.k if k is None else k
+    A, V = buf.A, buf.V
+    M = tr.M
+    B = tr.B
+    NO = M + 3 * k
+    dt = buf.latent.dtype
+    def outs():
+        d = dict(device="cuda")
+        return dict(S=torch.full((B, M), float("nan"), **d),
+                    sel=torch.full((B, max(k, 1)), -7, dtype=torch.int32, **d),
+                    mask=torch.full((B, M), 9, dtype=torch.uint8, **d),
+                    off=torch.full((B, M), -7, dtype=torch.int32, **d),
+                    mixed=torch.full((B, NO, tr.C * 4), float("nan"), dtype=dt, **d),
+                    pos=torch.full((B, NO, 2), -7, dtype=torch.int32, **d),
+                    span=torch.full((B, NO), -7, dtype=torch.int32, **d),
+                    src=torch.full((B, NO), -7, dtype=torch.int32, **d),
+                    sub=torch.full((B, NO), 9, dtype=torch.int8, **d))
+    a, f = outs(), outs()
+    av.avits_fuse_select(A, V, tr.alpha, k, a["sel"], a["off"], S=a["S"], sel_mask=a["mask"],
+                         perturb=perturb)
+    av.avits_selective_upsample(buf.latent, tr.frame_h, tr.frame_w, a["mask"], a["off"], k,
+                                a["mixed"], a["pos"], a["span"], a["src"], a["sub"],
+                                mode=buf.mode, pos_in=buf.pos_in, span_in=buf.span_in)
+    av.avits_select_upsample(A, V, tr.alpha, k, f["sel"], f["off"], f["mask"], buf.latent,
+                             tr.frame_h, tr.frame_w, f["mixed"], f["pos"], f["span"], f["src"],
+                             f["sub"], S=f["S"], perturb=perturb, mode=buf.mode,
+                             pos_in=buf.pos_in, span_in=buf.span_in)
+    assert _status(av) == 0
+    for key in a:
+        x, y = a[key], f[key]
+        if x.dtype in (torch.float32, torch.bfloat16):
+            x = x.view(torch.int32 if x.dtype == torch.float32 else torch.int16)
+            y = y.view(torch.int32 if y.dtype == torch.float32 else torch.int16)
+        if key == "sel" and k == 0:
+            continue
+        assert torch.equal(x, y), key
+
+
+@pytest.mark.parametrize("name,mode", [("tiny", "nearest"), ("flux1024", "nearest"),
+                                       ("flux1024", "bilinear"), ("batched", "nearest"),
+                                       ("flux2048", "nearest")])
+def test_select_upsample_fused_matches_separate(av, name, mode):
+    """One-launch selection + upsample (FLUX-2048: the two-kernel fallback)."""
+    from paper_2608_17995_gb300.pipeline import TransitionBuffers
+    from paper_2608_17995_gb300.workloads import make_transition
+    buf = TransitionBuffers(make_transition(name), mode=mode)
+    buf.spatial(); buf.temporal()
+    _fused_vs_separate(av, buf)
+
+
+def test_select_upsample_fused_edges(av):
+    """k = 0, k = M, ties with a perturbation, multi-level positions (the
+    batched schedule's second transition)."""
+    import torch
+    from paper_2608_17995_gb300.pipeline import TransitionBuffers
+    from paper_2608_17995_gb300.workloads import make_batched_stage2, make_transition
+    buf = TransitionBuffers(make_transition("flux1024"))
+    buf.spatial(); buf.temporal()
+    _fused_vs_separate(av, buf, k=0)
+    _fused_vs_separate(av, buf, k=buf.tr.M)
+    g = torch.Generator(device="cuda"); g.manual_seed(1)
+    pert = 1e-6 * torch.randn(buf.tr.B, buf.tr.M, device="cuda", generator=g)
+    _fused_vs_separate(av, buf, perturb=pert)
+    t1 = make_transition("batched")
+    b1 = TransitionBuffers(t1)
+    b1.run(merge=False)
+    t2 = make_batched_stage2(_np(b1.pos), _np(b1.span), frame=32, latent=_np(b1.mixed))
+    b2 = TransitionBuffers(t2)
+    b2.spatial(); b2.temporal()
+    _fused_vs_separate(av, b2)
+
+
 def test_batched_two_transitions(av, orc):
     """Batched multi-stage schedule: 8 elements, 16x16 -> 32x32 -> 64x64, the
     second transition re-scores every token of the mixed sequence, then the
