@@ -95,3 +95,39 @@ def test_product_path_does_not_touch_the_oracle():
             if f.endswith((".py", ".cu", ".cuh", ".h")):
                 text = open(os.path.join(dp, f)).read()
                 assert "import oracle" not in text and "avits_oracle" not in text, f
+
+
+def test_host_validation_of_the_extended_entry_points(lib):
+    """The perturbed selection, the key-mask spatial score and the fused
+    selection + upsample reject bad arguments on the host."""
+    P = ctypes.c_void_p(16)
+    INVALID, UNSUPPORTED = 1, 2
+    # perturbed selection: k > M, alpha outside [0,1] (the perturbation may be NULL)
+    assert lib.avits_fuse_select_perturbed(P, P, None, 1, 10, 0.5, 1e-6, 11, None, P, None, P,
+                                           None) == INVALID
+    assert lib.avits_fuse_select_perturbed(P, P, P, 1, 10, -0.1, 1e-6, 3, None, P, None, P,
+                                           None) == INVALID
+    # key mask: a NULL mask, Nk < M, non-positive scale
+    km = [P, P, 1, 1, 2, 64, 96, 64, 0, 0, 64, 0, 0, 64, None, 0.125, 1.0, 0, P, None, None, 0,
+          None]
+    assert lib.avits_score_spatial_keymask(*km) == INVALID
+    km[14] = P
+    km[6] = 32
+    assert lib.avits_score_spatial_keymask(*km) == INVALID
+    km[6] = 96
+    km[15] = 0.0
+    assert lib.avits_score_spatial_keymask(*km) == INVALID
+    # fused selection + upsample: the mask is required, k > M, patch size
+    # other than 2, bilinear on mixed-level input
+    su = [P, P, None, 1, 16, 0.5, 1e-6, 4, None, P, None, P, P, 1, 4, 4, 16, 2, None, None, 0,
+          P, P, P, P, P, None]
+    assert lib.avits_select_upsample(*su) == INVALID
+    su[10] = P
+    su[7] = 17
+    assert lib.avits_select_upsample(*su) == INVALID
+    su[7] = 4
+    su[17] = 3
+    assert lib.avits_select_upsample(*su) == UNSUPPORTED
+    su[17] = 2
+    su[18], su[19], su[20] = P, P, 1
+    assert lib.avits_select_upsample(*su) == UNSUPPORTED
