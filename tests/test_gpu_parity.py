@@ -149,17 +149,19 @@ def test_spatial_keymask_bf16(av, orc, B, H, M, Nk, d, kind):
 
 
 def test_spatial_keymask_first_l_is_l_form(av, orc):
-    """A mask of the first 512 keys (a multiple of the 64-key halves) takes
-    the same item paths as the L form: bit-identical A at the FLUX-1024 shape."""
+    """A mask of the first 384 keys (a multiple of the 64-key halves a
+    softmax warp reduces per item) takes the same item paths as the L form
+    with L = 384: bit-identical A at the FLUX-1024 shape."""
     import torch
     from paper_2608_17995_gb300.workloads import make_transition
     tr = make_transition("flux1024")
+    L = 384
     q, k = _dev(tr.q_img, "bf16"), _dev(tr.k_all, "bf16")
     A1 = torch.zeros(tr.B, tr.M, dtype=torch.float32, device="cuda")
     A2 = torch.zeros_like(A1)
-    av.avits_score_spatial(q, k, tr.L, tr.softmax_scale, A1)
+    av.avits_score_spatial(q, k, L, tr.softmax_scale, A1)
     mask = torch.zeros(tr.B, tr.Nk, dtype=torch.uint8, device="cuda")
-    mask[:, :tr.L] = 1
+    mask[:, :L] = 1
     av.avits_score_spatial(q, k, 0, tr.softmax_scale, A2, text_mask=mask)
     assert _status(av) == 0
     assert torch.equal(A1.view(torch.int32), A2.view(torch.int32))
