@@ -12,17 +12,27 @@
 //      an order-preserving 32-bit key (NaN -> 0, below everything; -0 -> +0;
 //      otherwise the IEEE bits with the sign bit flipped if positive, all
 //      bits flipped if negative), kept in registers and in shared memory;
-//   3. the k-th largest key by MSB-first radix select with 4-bit digits:
-//      each warp counts its keys per digit with ballots (lane j < 16 counts
-//      digit j; no shared-memory atomics, which would all hit one bin since
-//      scores in [0,1] share their top key bits), the per-warp counts go to a
-//      double-buffered table and every warp scans the 16 digits itself, so a
-//      pass costs one barrier; the passes stop once the k-th key's digit is
-//      taken whole;
-//   4. selection over contiguous per-thread index ranges with ONE block scan
-//      of (keys above the threshold, keys equal to it): the equal keys are
-//      taken lowest index first, so a thread's selected-before count is
-//      above_before + min(r, equal_before) for the r equal keys still needed;
+//   3. the k-th largest key.  Keys in registers: first one pass over 256
+//      buckets of the score VALUE (floor(256 S) clamped to [0, 255], a non-
+//      decreasing function of S, so of the key; scores in [0, 1] spread over
+//      the buckets where their top key bits do not), a shared-memory
+//      histogram and one block scan give the bucket holding the k-th key;
+//      when that bucket holds at most 32 keys one warp ranks them pairwise
+//      (key descending, index ascending) and the k-th is found.  Otherwise
+//      (clustered or tied scores), and for keys in shared memory: MSB-first
+//      radix select with 4-bit digits: each warp counts its keys per digit
+//      with ballots (lane j < 16 counts digit j; no shared-memory atomics,
+//      which would all hit one bin since the keys share their top bits), the
+//      per-warp counts go to a double-buffered table and every warp scans the
+//      16 digits itself, so a pass costs one barrier; the passes stop once
+//      the k-th key's digit is taken whole;
+//   4. the selection: keys above the threshold, and of the keys equal to it
+//      the lowest indices first.  Keys in registers: every key's selected-
+//      before count from per-warp ballots and one table of warp counts (one
+//      barrier), coalesced writes; keys in shared memory: contiguous per-
+//      thread index ranges with ONE block scan of (keys above, keys equal),
+//      a thread's selected-before count being above_before +
+//      min(r, equal_before) for the r equal keys still needed.  Either way
 //      it yields sel_idx (ascending), the mask and tok_offset.
 #include "avits_common.cuh"
 #include "avits_internal.h"
@@ -59,6 +69,59 @@ __device__ __forceinline__ uint32_t count_digits(uint32_t key, bool valid, uint3
   return __popc(m);
 }
 
+// Bucket of a fused score for the first selection pass: non-decreasing in S,
+// equal scores share a bucket, NaN (the lowest key) goes to bucket 0 and
+// scores outside [0, 1] (possible with a perturbation) to the end buckets.
+__device__ __forceinline__ int score_bucket(float s) {
+  if (s != s) return 0;
+  return (int)fminf(fmaxf(s * 256.0f, 0.0f), 255.0f);
+}
+
+// Block-wide prefix count of one flag per key, keys in registers (key
+// i = threadIdx.x + r * kThreads): before[r] = flagged keys of lower index;
+// returns the total.  `tab` holds R * kWarps words of shared memory; one
+// barrier, after which every warp scans the table of warp counts itself.
+template <int kThreads, int R>
+__device__ __forceinline__ uint32_t flag_prefix(const bool (&f)[R], uint32_t (&before)[R],
+                                                uint32_t* tab, int lane, int w) {
+  constexpr int kWarps = kThreads / 32;
+  constexpr int E = R * kWarps;           // table entries in (r, warp) order
+  constexpr int PER = (E + 31) / 32;      // entries per lane
+  uint32_t bal[R];
+#pragma unroll
+  for (int r = 0; r < R; ++r) bal[r] = __ballot_sync(0xffffffffu, f[r]);
+  if (lane == 0) {
+#pragma unroll
+    for (int r = 0; r < R; ++r) tab[r * kWarps + w] = __popc(bal[r]);
+  }
+  __syncthreads();
+  uint32_t loc[PER], sum = 0u;
+#pragma unroll
+  for (int j = 0; j < PER; ++j) {
+    const int e = lane * PER + j;
+    loc[j] = e < E ? tab[e] : 0u;
+    sum += loc[j];
+  }
+  uint32_t inc = sum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc += y;
+  }
+  const uint32_t excl = inc - sum;
+  const uint32_t lt = (1u << lane) - 1u;
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    // entry e of this warp's row r lives in lane e / PER, position e % PER
+    const int e = r * kWarps + w, src = e / PER, jj = e - src * PER;
+    uint32_t pre = excl;
+#pragma unroll
+    for (int j = 0; j < PER; ++j) pre += (j < jj) ? loc[j] : 0u;
+    before[r] = __shfl_sync(0xffffffffu, pre, src) + __popc(bal[r] & lt);
+  }
+  return __shfl_sync(0xffffffffu, inc, 31);
+}
+
 struct SelArgs {
   const float* A;
   const float* V;
@@ -75,7 +138,7 @@ struct SelArgs {
 
 // The selection of batch element b by one CTA.  kRegKeys keys per thread in
 // registers when M <= kRegKeys * kThreads; larger M (kRegKeys = 0) keeps them
-// in shared memory only.  `keys` is the CTA's dynamic shared memory (M words).
+// in shared memory only, in `keys` (the CTA's dynamic shared memory, M words).
 // write_out: this CTA writes S, sel_idx, the mask and tok_offset.  offs_s /
 // sel_s (or NULL): every token's start in the mixed sequence and whether it
 // is selected, left in shared memory for the fused upsample.
@@ -87,6 +150,13 @@ __device__ __forceinline__ void select_body(const SelArgs& g, int b, bool write_
   __shared__ uint32_t cnt[2][kWarps][16];
   __shared__ uint32_t scan_tot[kWarps];
   __shared__ int sh_nan;
+  __shared__ __align__(16) uint32_t hist[256];       // bucket counts (keys in registers)
+  __shared__ __align__(16) uint32_t cand_key[32];   // the k-th key's bucket, when small
+  __shared__ __align__(16) int cand_idx[32];
+  __shared__ uint32_t rank_part[8][32];  // candidate ranks, partial over 8 groups
+  __shared__ uint32_t sh_ncand;
+  __shared__ int sh_Tidx;
+  __shared__ uint32_t ptab[kRegKeys > 0 ? kRegKeys * kWarps : 1];   // flag_prefix table
   const float* __restrict__ A = g.A;
   const float* __restrict__ V = g.V;
   const float* __restrict__ perturb = g.perturb;
@@ -137,6 +207,10 @@ __device__ __forceinline__ void select_body(const SelArgs& g, int b, bool write_
   }
   if (lane == 0) { red[0][w] = amn; red[1][w] = amx; red[2][w] = vmn; red[3][w] = vmx; }
   if (tid == 0) sh_nan = 0;
+  if constexpr (in_regs) {
+    for (int j = tid; j < 256; j += kThreads) hist[j] = 0u;
+    if (tid == 0) sh_ncand = 0u;
+  }
   __syncthreads();
   {
     const bool in = lane < kWarps;
@@ -159,6 +233,7 @@ __device__ __forceinline__ void select_body(const SelArgs& g, int b, bool write_
   const float one_m = __fsub_rn(1.0f, alpha);
   int any_nan = 0;
   uint32_t rk[R];
+  int bk[R];
   auto fuse = [&](float x, float y, int i) {
     const float an = __fdiv_rn(__fsub_rn(x, amn), aden);
     const float vn = __fdiv_rn(__fsub_rn(y, vmn), vden);
@@ -170,12 +245,14 @@ __device__ __forceinline__ void select_body(const SelArgs& g, int b, bool write_
     for (int r = 0; r < R; ++r) {
       const int i = tid + r * kThreads;
       rk[r] = 0u;
+      bk[r] = -1;
       if (i < M) {
         const float s = fuse(ra[r], rv[r], i);
         if (S_out) S_out[(int64_t)b * M + i] = s;
         any_nan |= (s != s);
         rk[r] = order_key(s);
-        keys[i] = rk[r];
+        bk[r] = score_bucket(s);
+        atomicAdd(&hist[bk[r]], 1u);
       }
     }
   } else {
@@ -188,11 +265,107 @@ __device__ __forceinline__ void select_body(const SelArgs& g, int b, bool write_
   }
   if (any_nan) sh_nan = 1;
 
-  // 3. radix select of the k-th largest key
+  // 3. the k-th largest key: T on the top (32 - shift) key bits, of the keys
+  // whose prefix is T the `remaining` lowest indices are selected
   uint32_t prefix = 0u, pmask = 0u, remaining = (uint32_t)k;
   int shift = 32;
-  if (!in_regs) __syncthreads();   // keys are read back from shared memory below
-  if (k > 0 && k < M) {
+  bool radix = k > 0 && k < M;
+  uint32_t T = 0u;
+  uint32_t last_bin = 0u;   // keys with the k-th key's prefix (radix path)
+  int t_idx = 0x7fffffff;   // the last selected index among keys with prefix T
+  __syncthreads();   // histogram (keys in registers) or keys[] complete
+  if constexpr (in_regs) {
+    if (radix) {
+      // every warp scans the 256 bucket counts itself (no barrier): lane l
+      // holds buckets 255 - 8l - 7 .. 255 - 8l, taken in descending order
+      const uint4 h0 = *reinterpret_cast<const uint4*>(hist + 248 - 8 * lane);
+      const uint4 h1 = *reinterpret_cast<const uint4*>(hist + 252 - 8 * lane);
+      const uint32_t hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+      uint32_t lsum = 0u;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) lsum += hv[j];
+      uint32_t inc = lsum;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += y;
+      }
+      uint32_t cum = inc - lsum;
+      int my_bucket = -1;
+      uint32_t my_nb = 0u, my_above = 0u;
+#pragma unroll
+      for (int j = 7; j >= 0; --j) {
+        if (cum < (uint32_t)k && (uint32_t)k <= cum + hv[j]) {
+          my_bucket = 248 - 8 * lane + j;
+          my_nb = hv[j];
+          my_above = cum;
+        }
+        cum += hv[j];
+      }
+      const int src = __ffs(__ballot_sync(0xffffffffu, my_bucket >= 0)) - 1;
+      const int bucket = __shfl_sync(0xffffffffu, my_bucket, src);
+      const uint32_t nb = __shfl_sync(0xffffffffu, my_nb, src);
+      const uint32_t need = (uint32_t)k - __shfl_sync(0xffffffffu, my_above, src);   // 1..nb
+      if (nb <= 32u) {
+        radix = false;
+        // compaction of the bucket's keys: one shared-memory atomic per warp
+        bool in[R];
+        uint32_t bal[R], wcount = 0u;
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+          in[r] = bk[r] == bucket;
+          bal[r] = __ballot_sync(0xffffffffu, in[r]);
+          wcount += (uint32_t)__popc(bal[r]);
+        }
+        if (wcount != 0u) {
+          uint32_t base = 0u;
+          if (lane == 0) base = atomicAdd(&sh_ncand, wcount);
+          base = __shfl_sync(0xffffffffu, base, 0);
+          const uint32_t lt = (1u << lane) - 1u;
+#pragma unroll
+          for (int r = 0; r < R; ++r) {
+            if (in[r]) {
+              const uint32_t slot = base + __popc(bal[r] & lt);
+              cand_key[slot] = rk[r];
+              cand_idx[slot] = tid + r * kThreads;
+            }
+            base += (uint32_t)__popc(bal[r]);
+          }
+        }
+        __syncthreads();
+        // rank of candidate j = candidates above it (keys above, equal keys of
+        // lower index), the 32 x 32 comparisons spread over the CTA: thread
+        // (j = lane, g = warp < 8) compares candidate j with candidates
+        // 4g .. 4g + 3; every warp then sums the 8 partial counts itself
+        const bool have = (uint32_t)lane < nb;
+        const uint32_t kj = have ? cand_key[lane] : 0u;
+        const int ij = have ? cand_idx[lane] : 0;
+        if (w < 8) {
+          const int g0 = 4 * w;
+          uint32_t part = 0u;
+          if (have && (uint32_t)g0 < nb) {
+            const uint4 kv = *reinterpret_cast<const uint4*>(cand_key + g0);
+            const int4 iv = *reinterpret_cast<const int4*>(cand_idx + g0);
+            const uint32_t ka[4] = {kv.x, kv.y, kv.z, kv.w};
+            const int ia[4] = {iv.x, iv.y, iv.z, iv.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+              part += ((uint32_t)(g0 + e) < nb && (ka[e] > kj || (ka[e] == kj && ia[e] < ij))) ? 1u : 0u;
+          }
+          rank_part[w][lane] = part;
+        }
+        __syncthreads();
+        uint32_t rank = 0u;
+#pragma unroll
+        for (int g = 0; g < 8; ++g) rank += rank_part[g][lane];
+        const int kth = __ffs(__ballot_sync(0xffffffffu, have && rank == need - 1u)) - 1;
+        T = __shfl_sync(0xffffffffu, kj, kth);
+        t_idx = __shfl_sync(0xffffffffu, ij, kth);
+        shift = 0;
+      }
+    }
+  }
+  if (radix) {
     for (int pass = 0; pass < 8; ++pass) {
       shift -= 4;
       uint32_t c = 0;
@@ -235,16 +408,66 @@ __device__ __forceinline__ void select_body(const SelArgs& g, int b, bool write_
       prefix |= digit << shift;
       pmask |= 15u << shift;
       remaining = rem;
+      last_bin = bin;
       if (rem == bin) break;   // the digit is taken whole: no tie left to break
     }
+    T = prefix >> shift;
   }
-  // the selection is decided on the top (32 - shift) bits: keys whose prefix
-  // is above T are in; of the keys with prefix T the `remaining` lowest indices
-  const uint32_t T = shift < 32 ? (prefix >> shift) : 0u;
-  __syncthreads();   // keys[] complete for the range pass below
   if (write_out && tid == 0 && sh_nan) raise_status(g.status, AVITS_ERR_NAN);
 
-  // 4. one scan of (above, equal) over contiguous per-thread ranges
+  if constexpr (in_regs) {
+    // 4. keys in registers
+    const bool none = k == 0, all = k == M;
+    if (radix && remaining < last_bin) {
+      // radix path ending in equal keys: the index of the `remaining`-th
+      // lowest-index key with prefix T (a prefix count of the equal flags)
+      bool f[R];
+      uint32_t eb[R];
+#pragma unroll
+      for (int r = 0; r < R; ++r) f[r] = tid + r * kThreads < M && (rk[r] >> shift) == T;
+      flag_prefix<kThreads, R>(f, eb, ptab, lane, w);
+#pragma unroll
+      for (int r = 0; r < R; ++r)
+        if (f[r] && eb[r] == remaining - 1u) sh_Tidx = tid + r * kThreads;
+      __syncthreads();
+      t_idx = sh_Tidx;
+    }
+    bool f[R];
+    uint32_t before[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const int i = tid + r * kThreads;
+      bool sel = false;
+      if (i < M && !none) {
+        if (all) {
+          sel = true;
+        } else {
+          const uint32_t kp = rk[r] >> shift;
+          sel = kp > T || (kp == T && i <= t_idx);
+        }
+      }
+      f[r] = sel;
+    }
+    flag_prefix<kThreads, R>(f, before, ptab, lane, w);
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const int i = tid + r * kThreads;
+      if (i < M) {
+        const int c = (int)before[r];
+        if (write_out) {
+          tok_offset[(int64_t)b * M + i] = i + 3 * c;
+          if (mask) mask[(int64_t)b * M + i] = f[r] ? 1 : 0;
+          if (f[r]) sel_idx[(int64_t)b * k + c] = i;
+        }
+        if (offs_s) {
+          offs_s[i] = i + 3 * c;
+          sel_s[i] = f[r] ? 1 : 0;
+        }
+      }
+    }
+  } else {
+  // 4. keys in shared memory: one scan of (above, equal) over contiguous
+  // per-thread ranges
   const int per = (M + kThreads - 1) / kThreads;
   const int lo = min(M, tid * per), hi = min(M, lo + per);
   uint32_t gt = 0, eq = 0;
@@ -294,6 +517,7 @@ __device__ __forceinline__ void select_body(const SelArgs& g, int b, bool write_
       sel_s[i] = sel ? 1 : 0;
     }
     if (sel) ++c;
+  }
   }
 }
 

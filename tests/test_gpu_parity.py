@@ -398,6 +398,56 @@ def test_select_golden_ties_and_nan(av, orc):
     assert sel[0].tolist() == orc.topk(S, 3)[0][0].tolist() == [0, 2, 5]
 
 
+@pytest.mark.parametrize("n_bucket", [1, 31, 32, 33, 200])
+@pytest.mark.parametrize("ties", [False, True])
+def test_select_threshold_bucket_sizes(av, orc, n_bucket, ties):
+    """The k-th score inside a value bucket of width 1/256 holding n_bucket
+    scores: up to 32 they are ranked by one warp, beyond that the radix
+    select decides; ties inside the bucket take the lower index first."""
+    rng = np.random.default_rng(100 + n_bucket + 7 * ties)
+    B, M = 2, 1024
+    lo_b, hi_b = 100.0 / 256, 101.0 / 256
+    A = np.empty((B, M), np.float32)
+    for b in range(B):
+        rest = M - 2 - n_bucket
+        n_hi = rest // 3
+        below = rng.uniform(0.0, lo_b - 1e-3, rest - n_hi)
+        above = rng.uniform(hi_b + 1e-3, 1.0, n_hi)
+        inside = lo_b + 1e-3 + (hi_b - lo_b - 2e-3) * rng.uniform(0, 1, n_bucket)
+        if ties:
+            inside = np.round(inside * 4096) / 4096   # exact repeats within the bucket
+        vals = np.concatenate([[0.0, 1.0], below, above, inside]).astype(np.float32)
+        A[b] = vals[rng.permutation(M)]
+    k = 1 + (M - 2 - n_bucket) // 3 + (n_bucket + 1) // 2   # the k-th lands in the bucket
+    S, sel, mask, off, st = _run_select(av, A, np.zeros_like(A), 1.0, k)
+    assert st == 0
+    S_o = orc.fuse(A, np.zeros_like(A), 1.0)
+    assert np.array_equal(S.view(np.uint32), S_o.view(np.uint32))
+    kth = np.sort(S_o, axis=1)[:, ::-1][:, k - 1]
+    assert np.all(np.floor(kth * 256) == 100)
+    sel_o, mask_o, off_o = orc.topk(S_o, k)
+    assert np.array_equal(sel, sel_o)
+    assert np.array_equal(mask, mask_o)
+    assert np.array_equal(off, off_o)
+
+
+@pytest.mark.parametrize("M,k", [(1024, 307), (2048, 700), (4096, 1)])
+def test_select_clustered_scores(av, orc, M, k):
+    """Scores packed into one bucket apart from the two extremes: the radix
+    path over keys in registers, bit-exact."""
+    rng = np.random.default_rng(M + k)
+    A = (0.5 + 1e-4 * rng.standard_normal((2, M))).astype(np.float32)
+    A[:, 3] = 0.0
+    A[:, 7] = 1.0
+    S, sel, mask, off, st = _run_select(av, A, np.zeros_like(A), 1.0, k)
+    assert st == 0
+    S_o = orc.fuse(A, np.zeros_like(A), 1.0)
+    sel_o, mask_o, off_o = orc.topk(S_o, k)
+    assert np.array_equal(sel, sel_o)
+    assert np.array_equal(mask, mask_o)
+    assert np.array_equal(off, off_o)
+
+
 # ---------------------------------------------------- upsample / merge ----
 
 def _upsample(av, lat, dtype, gh, gw, mask, off, k, mode, pos_in=None, span_in=None):
