@@ -281,7 +281,7 @@ avits_status avits_selective_upsample(const void* latent, avits_dtype dt, int B,
  * launch (the transition of Sec. 3.2 after Eq. 8-9): every output is what
  * the two calls produce, bit for bit.  Each batch element gets several CTAs
  * that all compute its selection, so none waits for another; the first one
- * writes S_opt, sel_idx, sel_mask and tok_offset.  Up to M = 2048 tokens per
+ * writes S_opt, sel_idx, sel_mask and tok_offset.  Up to M = 4096 tokens per
  * element it is one kernel; above that the two kernels run back to back.
  * perturb : NULL or [B,M] fp32 (Eq. 9 tie-breaking noise, as
  *           avits_fuse_select_perturbed).

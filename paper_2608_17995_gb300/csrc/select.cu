@@ -1,6 +1,6 @@
 // select.cu — joint score and token selection (Sec. 3.3.3, Eq. 8-9).
 //
-// One CTA per batch element (256 threads up to M = 1024, 512 beyond; up to 8
+// One CTA per batch element (256 threads up to M = 256, 512 beyond; up to 8
 // keys per thread in registers), few barriers:
 //   1. min / max of A and V (NaN ignored): warp shuffles, one shared-memory
 //      round, every warp finishes the reduction itself;
@@ -604,16 +604,17 @@ cudaError_t launch_fuse_select(const float* A, const float* V, const float* pert
       if (dev >= 0 && dev < 64) __atomic_store_n(&done[dev], 1, __ATOMIC_RELEASE);
     }
   }
-  // 256 threads up to M = 1024 (fewer warps to synchronise and scan over,
-  // measured faster at FLUX-1024), 512 beyond; shared memory only above 4096
+  // 256 threads up to M = 256, 512 beyond (up to 2 keys per thread at
+  // FLUX-1024: the per-key work of the fuse step is the longest part, measured
+  // 3.50 -> 3.33 us against 256 threads); shared memory only above 4096
   void (*kern)(const SelArgs);
   int threads;
-  if (M <= 1024) {
+  if (M <= 256) {
     threads = 256;
-    const int per = (M + 255) / 256;
-    kern = per <= 1   ? fuse_select_kernel<256, 1>
-           : per <= 2 ? fuse_select_kernel<256, 2>
-                      : fuse_select_kernel<256, 4>;
+    kern = fuse_select_kernel<256, 1>;
+  } else if (M <= 1024) {
+    threads = kMaxThreads;
+    kern = M <= kMaxThreads ? fuse_select_kernel<kMaxThreads, 1> : fuse_select_kernel<kMaxThreads, 2>;
   } else {
     threads = kMaxThreads;
     const int per = (M + kMaxThreads - 1) / kMaxThreads;
@@ -622,8 +623,8 @@ cudaError_t launch_fuse_select(const float* A, const float* V, const float* pert
                                 : fuse_select_kernel<kMaxThreads, 0>;
   }
   cudaError_t ce = prefer_max_shared<fuse_select_kernel<256, 1>>();
-  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<256, 2>>();
-  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<256, 4>>();
+  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<kMaxThreads, 1>>();
+  if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<kMaxThreads, 2>>();
   if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<kMaxThreads, 4>>();
   if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<kMaxThreads, kMaxRegKeys>>();
   if (ce == cudaSuccess) ce = prefer_max_shared<fuse_select_kernel<kMaxThreads, 0>>();
@@ -636,9 +637,9 @@ cudaError_t launch_fuse_select(const float* A, const float* V, const float* pert
 
 namespace {
 
-constexpr int kFusedThreads = 256;
+constexpr int kFusedThreads = 512;
 constexpr int kFusedCtasTotal = 152;   // CTAs of the fused kernel over all elements
-constexpr int kFusedMaxM = kFusedThreads * kMaxRegKeys;   // 2048
+constexpr int kFusedMaxM = kFusedThreads * kMaxRegKeys;   // 4096
 
 template <typename T, bool kBilinear>
 cudaError_t launch_fused_t(const SelArgs& g, const UpsampleArgs<T>& u, int B, int M,
