@@ -13,8 +13,9 @@
 //   item  = (unit, 128-key tile)
 // The B*H*ceil(M/256)*ceil(Nk/128) items are split into equal contiguous
 // ranges, one per CTA, so every SM issues the same number of MMA tiles.  Every
-// (CTA, unit, softmax warpgroup) piece stores its per-row partial statistics
-// (max, sum over all keys, sum over text keys) in the workspace; a second,
+// (CTA, unit) piece stores its per-row partial statistics (max, sum over all
+// keys, sum over text keys; the two column halves merged in shared memory)
+// in the workspace; a second,
 // small kernel (spatial_finalize_kernel, launched as a programmatic dependent
 // of the first) merges the pieces of each (row, head) in slot order and sums
 // the heads in head order, so the result does not depend on CTA timing.
@@ -83,9 +84,13 @@ struct Bars {
   int abort;
 };
 
+// The column halves' row statistics meet here at the end of a segment: one
+// buffer per segment parity, per query tile, 128 rows x (m, la, lt).
+constexpr int kXchBytes = 2 * kQTiles * kBM * 3 * (int)sizeof(float);
+
 template <int D>
 constexpr int smem_bytes() {
-  return Cfg<D>::kQBytes + Cfg<D>::kKBytes + (int)sizeof(Bars) + 1024;
+  return Cfg<D>::kQBytes + Cfg<D>::kKBytes + (int)sizeof(Bars) + kXchBytes + 1024;
 }
 
 struct TcParams {
@@ -97,7 +102,7 @@ struct TcParams {
   int accumulate;
   float* A;
   float* lse;
-  float* part;      // [B*n_qp][H][2*max_parts][256][3]
+  float* part;      // [B*n_qp][H][max_parts][256][3]
   unsigned int* status;
   const uint8_t* tmask;   // [B,Nk] text-key mask, or NULL (text keys = the first L)
 };
@@ -486,6 +491,7 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
   uint8_t* sQ = smem;
   uint8_t* sK = smem + C::kQBytes;
   Bars* bars = reinterpret_cast<Bars*>(sK + C::kKBytes);
+  float* xch = reinterpret_cast<float*>(bars + 1);   // kXchBytes
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int it_begin = (int)blockIdx.x * p.per;
@@ -659,7 +665,7 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
     const int rowt = quad * 32 + lane;    // row within the tile
     const int rowu = t * kBM + rowt;      // row within the unit
     const uint32_t tlane = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(t * 2 * kBN + half * 64);
-    int li0 = 0;
+    int li0 = 0, sgi = 0;
     for (int it = it_begin; it < it_end;) {
       const Segment seg = segment_at(it, it_end, p.n_kt);
       RowStat st{-INFINITY, 0.f, 0.f};
@@ -706,13 +712,30 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
           if (lane == 0) mbar_arrive(&bars->s_empty[t][sb]);
         }
       }
-      // this warpgroup's piece of the unit: slot 2 * (CTA - first CTA of u) + half
-      const int u = seg.u;
-      const int slot = 2 * ((int)blockIdx.x - first_cta(u, p.n_kt, p.per)) + half;
-      float* pp = p.part + (((long long)u * (2 * p.max_parts) + slot) * kUnitRows + rowu) * 3;
-      pp[0] = st.m;
-      pp[1] = st.la;
-      pp[2] = st.lt;
+      // the two column halves of this tile's rows meet in shared memory
+      // (a buffer per segment parity, so one barrier per segment suffices);
+      // half 0 merges them and stores the CTA's piece of the unit, slot
+      // CTA - first CTA of u, which halves what the finalize kernel loads
+      float* xs = xch + (((sgi & 1) * kQTiles + t) * kBM + rowt) * 3;
+      if (half == 1) {
+        xs[0] = st.m;
+        xs[1] = st.la;
+        xs[2] = st.lt;
+      }
+      if (t == 0)   // the 8 softmax warps of query tile t (constant ids)
+        bar_sync(1, 8 * 32);
+      else
+        bar_sync(2, 8 * 32);
+      if (half == 0) {
+        merge_stat(st, xs[0], xs[1], xs[2]);
+        const int u = seg.u;
+        const int slot = (int)blockIdx.x - first_cta(u, p.n_kt, p.per);
+        float* pp = p.part + (((long long)u * p.max_parts + slot) * kUnitRows + rowu) * 3;
+        pp[0] = st.m;
+        pp[1] = st.la;
+        pp[2] = st.lt;
+      }
+      ++sgi;
       li0 += seg.nk;
       it += seg.nk;
     }
@@ -752,8 +775,8 @@ spatial_finalize_kernel(const TcParams p) {
   if (b < p.B) {
     for (int h = hl; h < p.H; h += kFinHeads) {
       const int u = (b * p.H + h) * p.n_qp + qp;
-      const int np = 2 * pieces(u, p.n_kt, p.per);
-      const float* q = p.part + ((long long)u * (2 * p.max_parts) * kUnitRows + rowu) * 3;
+      const int np = pieces(u, p.n_kt, p.per);
+      const float* q = p.part + ((long long)u * p.max_parts * kUnitRows + rowu) * 3;
       RowStat acc{-INFINITY, 0.f, 0.f};
       for (int s0 = 0; s0 < np; s0 += 6) {
         float v[6][3];
@@ -851,7 +874,7 @@ Plan make_plan(int B, int H, int M, int Nk, int num_sms) {
   if (pl.per < 1) pl.per = 1;
   pl.grid = (int)((pl.total + pl.per - 1) / pl.per);
   pl.max_parts = (int)((pl.n_kt + pl.per - 1) / pl.per) + 1;
-  pl.bytes = align256(sizeof(float) * 3 * (size_t)pl.n_units * 2 * pl.max_parts * kUnitRows);
+  pl.bytes = align256(sizeof(float) * 3 * (size_t)pl.n_units * pl.max_parts * kUnitRows);
   return pl;
 }
 
