@@ -326,6 +326,25 @@ size_t avits_merge_final_workspace(avits_upmode mode, int B, int full_h, int ful
  * ---------------------------------------------------------------------- */
 avits_status avits_device_status(void* stream);
 
+/* ------------------------------------------------------------------------
+ * Test hook for the failure detection of the device-side waits (a library
+ * facility; the paper has no counterpart).  Every spin in the kernels is an
+ * mbarrier wait bounded by a wall-clock limit: on expiry it records
+ * AVITS_ERR_TIMEOUT in the status word and raises its CTA's abort flag, which
+ * ends the waits of the other roles, and the kernel returns.  This call runs
+ * that code in one CTA on barriers nothing arrives at, so a test can exercise
+ * the path on a GPU without faulting it: warp 0 waits with `limit_ns`, warp 1
+ * waits on another barrier with 100 x limit_ns and gives up when warp 0
+ * raises the abort flag.
+ * limit_ns : 1e3 .. 1e8 (1 us .. 100 ms); else AVITS_ERR_INVALID_ARG.
+ * result   : device int64[5], written: [0] warp 0 completed (0 expected),
+ *            [1] warp 0's wait in ns, [2] warp 1 completed (0 expected),
+ *            [3] warp 1's wait in ns, [4] the abort flag (1 expected).
+ * The status word then holds AVITS_ERR_TIMEOUT (avits_device_status).
+ * ---------------------------------------------------------------------- */
+avits_status avits_selftest_bounded_wait(unsigned long long limit_ns, long long* result,
+                                         void* stream);
+
 /* Static text of a status code. */
 const char* avits_status_string(avits_status s);
 

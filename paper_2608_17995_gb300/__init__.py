@@ -29,7 +29,7 @@ __all__ = [
     "avits_score_spatiotemporal",
     "avits_score_temporal_var", "avits_fuse_select", "avits_selective_upsample",
     "avits_merge_final", "avits_merge_final_workspace", "avits_device_status",
-    "avits_status_string", "avits_version", "SpatialWorkspace",
+    "avits_selftest_bounded_wait", "avits_status_string", "avits_version", "SpatialWorkspace",
 ]
 
 F32, BF16 = 0, 1
@@ -86,6 +86,7 @@ def lib():
         "avits_merge_final": [vp, i32, i32, i32, vp, vp, i32, i32, i32, i32, i32, vp, vp, sz, vp],
         "avits_merge_final_workspace": [i32, i32, i32, i32],
         "avits_device_status": [vp],
+        "avits_selftest_bounded_wait": [ctypes.c_ulonglong, vp, vp],
         "avits_status_string": [i32],
         "avits_last_error_string": [],
         "avits_version": [],
@@ -152,6 +153,14 @@ def avits_status_string(code: int) -> str:
 def avits_device_status(stream=None) -> int:
     """Synchronise the stream; return and clear the device error code (0 = ok)."""
     return lib().avits_device_status(_stream(stream))
+
+
+def avits_selftest_bounded_wait(limit_ns: int, result, stream=None):
+    """Run the bounded-wait failure path on barriers nothing arrives at (a
+    test hook): result (cuda int64[5]) receives completion flags and wait
+    times of the timing-out warp and of the warp the abort flag releases."""
+    _check("avits_selftest_bounded_wait",
+           lib().avits_selftest_bounded_wait(int(limit_ns), _ptr(result), _stream(stream)))
 
 
 def avits_score_spatial_workspace(dtype, B, H, M, Nk, d) -> int:

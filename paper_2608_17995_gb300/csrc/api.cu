@@ -282,6 +282,14 @@ avits_status avits_merge_final(const void* mixed, avits_dtype dt, int B, int N, 
                                   workspace, status_word(), static_cast<cudaStream_t>(stream)));
 }
 
+avits_status avits_selftest_bounded_wait(unsigned long long limit_ns, long long* result,
+                                         void* stream) {
+  if (!result || limit_ns < 1000ull || limit_ns > 100ull * 1000ull * 1000ull)
+    return AVITS_ERR_INVALID_ARG;
+  return cuda_status(launch_wait_selftest(limit_ns, result, status_word(),
+                                          static_cast<cudaStream_t>(stream)));
+}
+
 avits_status avits_device_status(void* stream) {
   cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_status(e);

@@ -78,17 +78,19 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
 
 // Wait for the phase of `bar` with the given parity to complete.  Gives up
 // when *abort_flag becomes non-zero (another role timed out; pass nullptr to
-// ignore it) or after the time / iteration limit, in which case it raises
-// AVITS_ERR_TIMEOUT and sets *abort_flag.  Returns true on completion.
+// ignore it) or after the time limit (limit_ns, 1 s by default) or the
+// iteration cap, in which case it raises AVITS_ERR_TIMEOUT and sets
+// *abort_flag.  Returns true on completion.
 __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity,
-                                                  volatile int* abort_flag, unsigned int* st) {
+                                                  volatile int* abort_flag, unsigned int* st,
+                                                  unsigned long long limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = globaltimer_ns();
   for (unsigned long long it = 1; it < kWaitMaxIters; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 63ull) == 0) {
       if (abort_flag && *abort_flag) return false;
-      if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+      if (globaltimer_ns() - t0 > limit_ns) break;
     }
   }
   raise_status(st, AVITS_ERR_TIMEOUT);

@@ -43,6 +43,10 @@ cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s,
 cudaError_t launch_spatial_simt(const SpatialArgs& a, cudaStream_t s);
 
 // ---- temporal ---------------------------------------------------------------
+// Failure-detection test hook (selftest.cu): bounded waits that cannot complete.
+cudaError_t launch_wait_selftest(unsigned long long limit_ns, long long* result,
+                                 unsigned int* status, cudaStream_t s);
+
 cudaError_t launch_temporal(const void* ht, const void* hp, avits_dtype dt, int B, int N, int D,
                             float eps, float* V, int num_sms, unsigned int* status, cudaStream_t s);
 // The temporal score as a programmatic dependent of the kernel just launched

@@ -131,3 +131,14 @@ def test_host_validation_of_the_extended_entry_points(lib):
     su[17] = 2
     su[18], su[19], su[20] = P, P, 1
     assert lib.avits_select_upsample(*su) == UNSUPPORTED
+
+
+def test_host_validation_of_the_wait_selftest(lib):
+    """The failure-detection test hook rejects a missing result buffer and
+    limits outside 1 us .. 100 ms before launching anything."""
+    P = ctypes.c_void_p(16)
+    f = lib.avits_selftest_bounded_wait
+    assert f(ctypes.c_ulonglong(1000000), None, None) == 1
+    assert f(ctypes.c_ulonglong(0), P, None) == 1
+    assert f(ctypes.c_ulonglong(999), P, None) == 1
+    assert f(ctypes.c_ulonglong(100000001), P, None) == 1
