@@ -10,6 +10,8 @@
 // the half-pixel-centred 2x bilinear resize of the rebuilt low-res grid, in
 // which each 2x2 block of span-1 tokens contributes its 2x2 average pools.
 // Algorithmic bytes: B*N*(T*elt + 12) read + B*fh*fw*T*elt written.
+#include <algorithm>
+
 #include "avits_common.cuh"
 #include "avits_internal.h"
 
@@ -68,9 +70,22 @@ merge_nearest_kernel(const T* __restrict__ mixed, int B, int N, const int32_t* _
   }
 }
 
+// Cell map entry: the covering token's index, with kSpan2 set when its span
+// is 2 (the gather then needs no span lookup); -1 = a hole.
+constexpr int32_t kSpan2 = 1 << 30;
+
+// The cell map starts as -1 everywhere (a hole until a token claims it).
+__global__ void merge_fill_kernel(int32_t* __restrict__ map, int64_t n) {
+  pdl_wait_then_trigger();
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    map[i] = -1;
+}
+
 __global__ void merge_map_kernel(int B, int N, const int32_t* __restrict__ pos,
                                  const int32_t* __restrict__ span, int fh, int fw,
                                  int32_t* __restrict__ map, unsigned int* status) {
+  pdl_wait_then_trigger();
   const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= (int64_t)B * N) return;
   const int b = (int)(t / N), ti = (int)(t % N);
@@ -80,42 +95,43 @@ __global__ void merge_map_kernel(int B, int N, const int32_t* __restrict__ pos,
     raise_status(status, AVITS_ERR_COVERAGE);
     return;
   }
+  const int32_t entry = ti | (s == 2 ? kSpan2 : 0);
   for (int u = 0; u < s; ++u)
     for (int v = 0; v < s; ++v) {
-      const int old = atomicExch(&map[(int64_t)b * fh * fw + (int64_t)(y + u) * fw + x + v], ti);
+      const int old = atomicExch(&map[(int64_t)b * fh * fw + (int64_t)(y + u) * fw + x + v], entry);
       if (old != -1) raise_status(status, AVITS_ERR_COVERAGE);
     }
 }
 
+// Low-resolution pixel (r, c) of the rebuilt grid from the map entries of its
+// even-aligned cell (e0) and of its own cell (e1): a span-2 token gives its
+// patch pixel, a span-1 token its 2x2 average pool ((a+b)+(c+d))/4; 0 for a
+// hole (already reported).
 template <typename T>
-__device__ __forceinline__ float low_pixel(const T* __restrict__ mb, const int32_t* __restrict__ mapb,
-                                           const int32_t* __restrict__ spanb, int fw, int T4, int ch,
-                                           int r, int c) {
-  const int t0 = mapb[(r & ~1) * fw + (c & ~1)];
-  if (t0 < 0) return 0.f;
-  if (spanb[t0] == 2) return load_elem(mb, (int64_t)t0 * T4 + ch * 4 + (r & 1) * 2 + (c & 1));
-  const int t1 = mapb[r * fw + c];
-  if (t1 < 0) return 0.f;
-  const T* p = mb + (int64_t)t1 * T4 + ch * 4;
+__device__ __forceinline__ float low_value(const T* __restrict__ mb, int T4, int ch, int r, int c,
+                                           int32_t e0, int32_t e1) {
+  if (e0 < 0) return 0.f;
+  if (e0 & kSpan2)
+    return load_elem(mb, (int64_t)(e0 & ~kSpan2) * T4 + ch * 4 + (r & 1) * 2 + (c & 1));
+  if (e1 < 0) return 0.f;
+  const T* p = mb + (int64_t)(e1 & ~kSpan2) * T4 + ch * 4;
   const float top = __fadd_rn(load_elem(p, 0), load_elem(p, 1));
   const float bot = __fadd_rn(load_elem(p, 2), load_elem(p, 3));
   return __fmul_rn(__fadd_rn(top, bot), 0.25f);
 }
 
-__device__ __forceinline__ void bil_axis(int P, int n, int& r0, int& r1, float& w0, float& w1) {
-  const int m = P >> 1;
-  if ((P & 1) == 0) { r0 = m - 1; r1 = m; w0 = 0.25f; w1 = 0.75f; }
-  else { r0 = m; r1 = m + 1; w0 = 0.75f; w1 = 0.25f; }
-  r0 = max(r0, 0);
-  r1 = min(r1, n - 1);
-}
-
+// One thread per (output cell, channel).  A span-2 cell's four pixels draw on
+// the 3 x 3 low-resolution neighbourhood around it; all map entries of that
+// neighbourhood are loaded first, then all pixel values, so the chains of
+// dependent loads are two deep.
 template <typename T>
 __global__ void merge_bilinear_kernel(const T* __restrict__ mixed, int B, int N,
                                       const int32_t* __restrict__ span, int fh, int fw, int C,
                                       const int32_t* __restrict__ map, T* __restrict__ out,
                                       unsigned int* status) {
   using PV = typename Pix4<T>::V;
+  pdl_wait_then_trigger();
+  (void)span;
   const int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t cells = (int64_t)fh * fw;
   if (g >= (int64_t)B * cells * C) return;
@@ -126,30 +142,49 @@ __global__ void merge_bilinear_kernel(const T* __restrict__ mixed, int B, int N,
   const int Y = cell / fw, X = cell - Y * fw;
   const int T4 = C * 4;
   const int32_t* mapb = map + (int64_t)b * cells;
-  const int32_t* spanb = span + (int64_t)b * N;
   const T* mb = mixed + (int64_t)b * N * T4;
-  const int t = mapb[cell];
+  const int32_t e = mapb[cell];
   PV* dst = reinterpret_cast<PV*>(out + bc * T4) + c;
-  if (t < 0) {
+  if (e < 0) {
     raise_status(status, AVITS_ERR_COVERAGE);
     *dst = Pix4<T>::make(0.f, 0.f, 0.f, 0.f);
     return;
   }
-  if (spanb[t] == 1) {
-    *dst = reinterpret_cast<const PV*>(mb + (int64_t)t * T4)[c];
+  if (!(e & kSpan2)) {
+    *dst = reinterpret_cast<const PV*>(mb + (int64_t)e * T4)[c];
     return;
   }
+  // rows and columns of the neighbourhood (clamped to the frame)
+  int rr[3], cc[3];
+#pragma unroll
+  for (int k = 0; k < 3; ++k) {
+    rr[k] = min(max(Y - 1 + k, 0), fh - 1);
+    cc[k] = min(max(X - 1 + k, 0), fw - 1);
+  }
+  int32_t e0[3][3], e1[3][3];
+#pragma unroll
+  for (int i = 0; i < 3; ++i)
+#pragma unroll
+    for (int j = 0; j < 3; ++j) {
+      e0[i][j] = mapb[(rr[i] & ~1) * fw + (cc[j] & ~1)];
+      e1[i][j] = mapb[rr[i] * fw + cc[j]];
+    }
+  float lv[3][3];
+#pragma unroll
+  for (int i = 0; i < 3; ++i)
+#pragma unroll
+    for (int j = 0; j < 3; ++j) lv[i][j] = low_value(mb, T4, c, rr[i], cc[j], e0[i][j], e1[i][j]);
   float r[4];
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
-    int r0, r1, c0, c1;
-    float wy0, wy1, wx0, wx1;
-    bil_axis(2 * Y + (q >> 1), fh, r0, r1, wy0, wy1);
-    bil_axis(2 * X + (q & 1), fw, c0, c1, wx0, wx1);
-    const float p00 = low_pixel(mb, mapb, spanb, fw, T4, c, r0, c0);
-    const float p01 = low_pixel(mb, mapb, spanb, fw, T4, c, r0, c1);
-    const float p10 = low_pixel(mb, mapb, spanb, fw, T4, c, r1, c0);
-    const float p11 = low_pixel(mb, mapb, spanb, fw, T4, c, r1, c1);
+    // output pixel row 2Y + a draws on rows (Y - 1, Y) for a = 0 and (Y, Y + 1)
+    // for a = 1 with weights (1/4, 3/4) / (3/4, 1/4), clamped at the frame
+    // edge: neighbourhood rows a and a + 1; columns likewise
+    const int a = q >> 1, bq = q & 1;
+    const float wy0 = a ? 0.75f : 0.25f, wy1 = a ? 0.25f : 0.75f;
+    const float wx0 = bq ? 0.75f : 0.25f, wx1 = bq ? 0.25f : 0.75f;
+    const float p00 = lv[a][bq], p01 = lv[a][bq + 1];
+    const float p10 = lv[a + 1][bq], p11 = lv[a + 1][bq + 1];
     const float top = __fadd_rn(__fmul_rn(wx0, p00), __fmul_rn(wx1, p01));
     const float bot = __fadd_rn(__fmul_rn(wx0, p10), __fmul_rn(wx1, p11));
     r[q] = __fadd_rn(__fmul_rn(wy0, top), __fmul_rn(wy1, bot));
@@ -172,16 +207,27 @@ cudaError_t launch_t(const void* mixed, int B, int N, const int32_t* pos, const 
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
   }
+  // three kernels (fill, scatter of the cell map, gather), each a
+  // programmatic dependent of the one before: their launches overlap, every
+  // kernel waits for its predecessor before touching memory
   int32_t* map = static_cast<int32_t*>(ws);
-  cudaError_t e = cudaMemsetAsync(map, 0xFF, sizeof(int32_t) * (size_t)B * fh * fw, s);
+  const int64_t ncell = (int64_t)B * fh * fw;
+  cudaError_t e = prefer_max_shared<merge_fill_kernel>();
+  if (e == cudaSuccess) e = prefer_max_shared<merge_map_kernel>();
+  if (e == cudaSuccess) e = prefer_max_shared<merge_bilinear_kernel<T>>();
+  if (e != cudaSuccess) return e;
+  const int fill_grid = (int)std::min<int64_t>((ncell + 255) / 256, 1024);
+  e = launch_pdl(merge_fill_kernel, dim3(fill_grid), dim3(256), 0, s, map, ncell);
   if (e != cudaSuccess) return e;
   const int64_t nt = (int64_t)B * N;
-  merge_map_kernel<<<(int)((nt + 255) / 256), 256, 0, s>>>(B, N, pos, span, fh, fw, map, status);
-  e = cudaGetLastError();
+  e = launch_pdl(merge_map_kernel, dim3((unsigned)((nt + 255) / 256)), dim3(256), 0, s, B, N, pos,
+                 span, fh, fw, map, status);
   if (e != cudaSuccess) return e;
   const int64_t work = (int64_t)B * fh * fw * C;
-  merge_bilinear_kernel<T><<<(int)((work + 255) / 256), 256, 0, s>>>(
-      static_cast<const T*>(mixed), B, N, span, fh, fw, C, map, static_cast<T*>(out), status);
+  e = launch_pdl(merge_bilinear_kernel<T>, dim3((unsigned)((work + 255) / 256)), dim3(256), 0, s,
+                 static_cast<const T*>(mixed), B, N, span, fh, fw, C,
+                 static_cast<const int32_t*>(map), static_cast<T*>(out), status);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
