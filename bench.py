@@ -365,6 +365,7 @@ def run_ours(args, world, rank, local, pg):
         result["batched_schedule"] = batched_schedule_measure(torch, av, dev, stream, K)
         result["temporal_var"] = temporal_var_measure(torch, av, tr, dev, stream, peaks)
         result["spatial_keymask"] = keymask_measure(torch, av, buf, tr, sets, nsets, stream, peaks)
+        result["spatial_from_lse"] = lse_measure(torch, av, buf, tr, sets, nsets, stream, peaks)
     return result, tr
 
 
@@ -523,6 +524,29 @@ def keymask_measure(torch, av, buf, tr, sets, nsets, stream, peaks):
                      "text_keys": int(m.sum())}
     out["status"] = av.avits_device_status(stream)
     return out
+
+
+def lse_measure(torch, av, buf, tr, sets, nsets, stream, peaks):
+    """avits_score_spatial_lse at the FLUX-1024 shape: the text mass from the
+    caller's logsumexp over all keys (as a model's attention forward returns
+    it) and the L = 512 text keys only, rotated over the same input copies."""
+    A = torch.empty(tr.B, tr.M, dtype=torch.float32, device=buf.A.device)
+    lse = torch.empty(tr.B, tr.H, tr.M, 2, dtype=torch.float32, device=buf.A.device)
+    av.avits_score_spatial(sets[0][0], sets[0][1], tr.L, tr.softmax_scale, A, lse=lse,
+                           workspace=buf.ws, stream=stream)
+    lse_all = lse[..., 0].contiguous()
+
+    def fn():
+        for s_ in range(nsets):
+            av.avits_score_spatial_lse(sets[s_][0], sets[s_][1][:, :, :tr.L], lse_all,
+                                       tr.softmax_scale, A, workspace=buf.ws, stream=stream)
+
+    ms = _graph_time_ms(torch, stream, fn, 20) / nsets
+    flops = 2.0 * tr.B * tr.H * tr.M * tr.L * tr.d
+    tf = flops / (ms * 1e-3) / 1e12
+    return {"us": round(ms * 1e3, 3), "tflops": round(tf, 2),
+            "frac_tensor": round(tf / peaks["bf16_tflops"], 4), "text_keys": tr.L,
+            "status": av.avits_device_status(stream)}
 
 
 def temporal_var_measure(torch, av, tr, dev, stream, peaks, n_t=4, n_sets=6):

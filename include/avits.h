@@ -146,6 +146,31 @@ size_t avits_score_spatial_noalloc_limit(void);
 const char* avits_score_spatial_noalloc_error(void);
 
 /* ------------------------------------------------------------------------
+ * avits_score_spatial when the caller already has the logsumexp over ALL
+ * keys, e.g. from the model's own joint-attention forward (fused attention
+ * returns it; Sec. 3.3.1 recomputes the attention only because fused
+ * kernels do not expose the weights).  Eq. 5's text mass is
+ * exp(lse_txt - lse_all), so only the L text keys are scored here: a third
+ * of the key work at FLUX-1024 (L = 512 of Nk = 1536).
+ * k_txt   : [B,H,L,d] the text keys (e.g. the first L rows of k_all, with
+ *           k_all's strides).  q_img, dt, strides, softmax_scale, weight,
+ *           accumulate and A as avits_score_spatial.
+ * lse_all : [B,H,M] fp32, contiguous: natural-log logsumexp of s*q_i.k_j over
+ *           every key of the joint sequence, for the same s and the same
+ *           queries.  Inconsistent values give masses outside [0, 1].
+ * lse_opt : NULL or [B,H,M,2]: (lse_all as given, lse_txt).
+ * workspace : avits_score_spatial_workspace(dt, B, H, M, L, d) bytes.
+ * Tensor-core path only (bf16, d in {64,128}, 16-byte aligned layout);
+ * anything else returns AVITS_ERR_UNSUPPORTED.
+ * ---------------------------------------------------------------------- */
+avits_status avits_score_spatial_lse(const void* q_img, const void* k_txt, avits_dtype dt,
+                                     int B, int H, int M, int L, int d, int64_t q_sb,
+                                     int64_t q_sh, int64_t q_sn, int64_t k_sb, int64_t k_sh,
+                                     int64_t k_sn, const float* lse_all, float softmax_scale,
+                                     float weight, int accumulate, float* A, float* lse_opt,
+                                     void* workspace, size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
  * avits_score_spatial for sequences whose text and image tokens interleave
  * (the unified sequences of MLLM-conditioned models, Sec. 3.3.1): the text
  * keys are the keys j with text_mask[b*Nk + j] != 0 instead of the first L.

@@ -25,7 +25,8 @@ from . import _build
 
 __all__ = [
     "AvitsError", "build", "lib", "library_path",
-    "avits_score_spatial", "avits_score_spatial_workspace", "avits_score_temporal",
+    "avits_score_spatial", "avits_score_spatial_workspace", "avits_score_spatial_lse",
+    "avits_score_temporal",
     "avits_score_spatiotemporal",
     "avits_score_temporal_var", "avits_fuse_select", "avits_selective_upsample",
     "avits_merge_final", "avits_merge_final_workspace", "avits_device_status",
@@ -72,6 +73,8 @@ def lib():
         "avits_score_spatial_workspace": [i32, i32, i32, i32, i32, i32],
         "avits_score_spatial_keymask": [vp, vp, i32, i32, i32, i32, i32, i32, i64, i64, i64, i64,
                                         i64, i64, vp, f32, f32, i32, vp, vp, vp, sz, vp],
+        "avits_score_spatial_lse": [vp, vp, i32, i32, i32, i32, i32, i32, i64, i64, i64, i64,
+                                    i64, i64, vp, f32, f32, i32, vp, vp, vp, sz, vp],
         "avits_score_temporal": [vp, vp, i32, i32, i32, i32, f32, vp, vp],
         "avits_score_spatiotemporal": [vp, vp, i32, i32, i32, i32, i32, i32, i32, i64, i64, i64,
                                        i64, i64, i64, f32, f32, i32, vp, vp, vp, sz, vp, vp, i32,
@@ -233,6 +236,39 @@ def avits_score_spatial(q_img, k_all, L: int, softmax_scale: float, A, weight: f
         float(softmax_scale), float(weight), 1 if accumulate else 0,
         _ptr(A), _ptr(lse), _ptr(wbuf), wbytes, _stream(stream))
     _check("avits_score_spatial", rc)
+    return A
+
+
+def avits_score_spatial_lse(q_img, k_txt, lse_all, softmax_scale: float, A, weight: float = 1.0,
+                            accumulate: bool = False, lse=None,
+                            workspace: Optional[SpatialWorkspace] = None, stream=None):
+    """Eq. 5 from the caller's logsumexp over all keys: q_img [B,H,M,d],
+    k_txt [B,H,L,d] (the text keys only, any strides with d contiguous),
+    lse_all [B,H,M] fp32 contiguous (natural log, e.g. from the model's
+    attention forward); A [B,M] written (or accumulated)."""
+    B, H, M, d = q_img.shape
+    L = k_txt.shape[2]
+    if k_txt.shape[0] != B or k_txt.shape[1] != H or k_txt.shape[3] != d:
+        raise ValueError("q_img / k_txt shapes disagree")
+    if q_img.stride(3) != 1 or k_txt.stride(3) != 1:
+        raise ValueError("the head-dim axis must be contiguous")
+    if tuple(lse_all.shape) != (B, H, M) or not lse_all.is_contiguous():
+        raise ValueError("lse_all must be a contiguous [B,H,M] tensor")
+    dt = _dtype_code(q_img)
+    if _dtype_code(k_txt) != dt:
+        raise TypeError("q_img and k_txt dtypes differ")
+    need = int(lib().avits_score_spatial_workspace(dt, B, H, M, L, d))
+    if workspace is None:
+        key = (q_img.device.index, _torch().cuda.current_stream().cuda_stream if stream is None else _stream(stream))
+        workspace = _default_ws.setdefault(key, SpatialWorkspace(q_img.device))
+    wbuf, wbytes = workspace.get(need)
+    rc = lib().avits_score_spatial_lse(
+        _ptr(q_img), _ptr(k_txt), dt, B, H, M, L, d,
+        q_img.stride(0), q_img.stride(1), q_img.stride(2),
+        k_txt.stride(0), k_txt.stride(1), k_txt.stride(2), _ptr(lse_all),
+        float(softmax_scale), float(weight), 1 if accumulate else 0,
+        _ptr(A), _ptr(lse), _ptr(wbuf), wbytes, _stream(stream))
+    _check("avits_score_spatial_lse", rc)
     return A
 
 

@@ -110,6 +110,28 @@ avits_status avits_score_spatial(const void* q_img, const void* k_all, avits_dty
   return cuda_status(launch_spatial_simt(a, s));
 }
 
+avits_status avits_score_spatial_lse(const void* q_img, const void* k_txt, avits_dtype dt, int B,
+                                     int H, int M, int L, int d, int64_t q_sb, int64_t q_sh,
+                                     int64_t q_sn, int64_t k_sb, int64_t k_sh, int64_t k_sn,
+                                     const float* lse_all, float softmax_scale, float weight,
+                                     int accumulate, float* A, float* lse_opt, void* workspace,
+                                     size_t ws_bytes, void* stream) {
+  if (!q_img || !k_txt || !lse_all || !A || !valid_dtype(dt)) return AVITS_ERR_INVALID_ARG;
+  if (B <= 0 || H <= 0 || M <= 0 || L <= 0 || d <= 0) return AVITS_ERR_INVALID_ARG;
+  if (!(softmax_scale > 0.f) || !(softmax_scale < 3.0e38f)) return AVITS_ERR_INVALID_ARG;
+  if (q_sn < d || k_sn < d || q_sh < 0 || k_sh < 0 || q_sb < 0 || k_sb < 0)
+    return AVITS_ERR_INVALID_ARG;
+  SpatialArgs a{q_img, k_txt, dt, B, H, M, L, L, d, q_sb, q_sh, q_sn, k_sb, k_sh, k_sn,
+                softmax_scale, weight, accumulate ? 1 : 0, A, lse_opt, workspace, ws_bytes,
+                status_word()};
+  a.lse_all = lse_all;
+  if (!spatial_tc_eligible(a)) return AVITS_ERR_UNSUPPORTED;
+  const int sms = num_sms_current();
+  if (ws_bytes < spatial_tc_workspace(B, H, M, L, d, sms) || !workspace)
+    return AVITS_ERR_INVALID_ARG;
+  return cuda_status(launch_spatial_tc(a, sms, static_cast<cudaStream_t>(stream)));
+}
+
 avits_status avits_score_spatial_keymask(const void* q_img, const void* k_all, avits_dtype dt,
                                          int B, int H, int M, int Nk, int d, int64_t q_sb,
                                          int64_t q_sh, int64_t q_sn, int64_t k_sb, int64_t k_sh,

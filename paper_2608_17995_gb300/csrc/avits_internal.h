@@ -28,6 +28,10 @@ struct SpatialArgs {
   size_t ws_bytes;
   unsigned int* status;
   const uint8_t* tmask = nullptr;   // [B,Nk], nonzero = text key; NULL: keys j < L
+  // [B,H,M] natural-log logsumexp over ALL keys, computed by the caller (the
+  // model's attention forward); then the keys given are the text keys only
+  // and the mass is exp(lse_txt - lse_all).  NULL: the keys are all keys.
+  const float* lse_all = nullptr;
 };
 
 // tcgen05 / TMA path (bf16, d in {64,128}); returns false if the shape or

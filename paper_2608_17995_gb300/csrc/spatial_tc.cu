@@ -105,6 +105,7 @@ struct TcParams {
   float* part;      // [B*n_qp][H][max_parts][256][3]
   unsigned int* status;
   const uint8_t* tmask;   // [B,Nk] text-key mask, or NULL (text keys = the first L)
+  const float* lse_all;   // [B,H,M] caller's logsumexp over all keys (natural log), or NULL
 };
 
 // ------------------------------------------------------------------ PTX ----
@@ -792,11 +793,28 @@ spatial_finalize_kernel(const TcParams p) {
         for (int k = 0; k < 6; ++k)
           if (s0 + k < np) merge_stat(acc, v[k][0], v[k][1], v[k][2]);
       }
-      sum += acc.lt / acc.la;
-      if (p.lse && row < p.M) {
-        float* lp = p.lse + (((long long)b * p.H + h) * p.M + row) * 2;
-        lp[0] = (acc.m + __log2f(acc.la)) * ln2;
-        lp[1] = acc.lt > 0.f ? (acc.m + __log2f(acc.lt)) * ln2 : -INFINITY;
+      if (p.lse_all) {
+        // the keys of this pass are the text keys only: mass = exp(lse_txt -
+        // lse_all) against the caller's logsumexp over all keys
+        float ratio = 0.f;
+        if (row < p.M) {
+          const float la_all = p.lse_all[((long long)b * p.H + h) * p.M + row];
+          ratio = acc.lt > 0.f ? exp2f(acc.m + log2f(acc.lt) - la_all * 1.4426950408889634f)
+                               : 0.f;
+          if (p.lse) {
+            float* lp = p.lse + (((long long)b * p.H + h) * p.M + row) * 2;
+            lp[0] = la_all;
+            lp[1] = acc.lt > 0.f ? (acc.m + log2f(acc.lt)) * ln2 : -INFINITY;
+          }
+        }
+        sum += ratio;
+      } else {
+        sum += acc.lt / acc.la;
+        if (p.lse && row < p.M) {
+          float* lp = p.lse + (((long long)b * p.H + h) * p.M + row) * 2;
+          lp[0] = (acc.m + __log2f(acc.la)) * ln2;
+          lp[1] = acc.lt > 0.f ? (acc.m + __log2f(acc.lt)) * ln2 : -INFINITY;
+        }
       }
     }
   }
@@ -955,6 +973,7 @@ cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s,
   p.part = reinterpret_cast<float*>(ws);
   p.status = a.status;
   p.tmask = a.tmask;
+  p.lse_all = a.lse_all;
   cudaError_t e = set_smem_once();
   if (e != cudaSuccess) return e;
   const bool masked = p.tmask != nullptr;

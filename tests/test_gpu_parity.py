@@ -85,6 +85,55 @@ def _check_spatial(av, orc, q, k, L, scale, dtype, rows=None, rtol=BF16_RTOL, we
     return A_g
 
 
+@pytest.mark.parametrize("name,nrows", [("tiny", None), ("flux1024", 40), ("edit", 24), ("batched", 32)])
+def test_spatial_from_lse_all(av, orc, name, nrows):
+    """Eq. 5 from the logsumexp over all keys (as a model's attention forward
+    returns it) and the text keys only: A against the oracle on the same
+    rows, lse_all taken from the oracle (fp64 rounded to fp32)."""
+    import torch
+    from paper_2608_17995_gb300.workloads import make_transition, to_bf16_bits
+    tr = make_transition(name)
+    q, k = tr.q_img, tr.k_all
+    if q.dtype == np.float32:   # the fp32 config: the same bf16 values on both sides
+        q, k = to_bf16_bits(q), to_bf16_bits(k)
+    B, H, M, d = q.shape
+    rows = None if nrows is None else _sample_rows(B, M, nrows, seed=3)
+    A_o, mass_o, lse_o = orc.score_spatial(q, k, tr.L, tr.softmax_scale, rows=rows)
+    lse_all = torch.from_numpy(np.ascontiguousarray(lse_o[..., 0].astype(np.float32))).cuda()
+    qd, kd = _dev(q, "bf16"), _dev(k, "bf16")
+    A = torch.zeros(B, M, dtype=torch.float32, device="cuda")
+    lse = torch.zeros(B, H, M, 2, dtype=torch.float32, device="cuda")
+    av.avits_score_spatial_lse(qd, kd[:, :, :tr.L], lse_all, tr.softmax_scale, A, lse=lse)
+    assert _status(av) == 0
+    idx = np.arange(B * M) if rows is None else np.asarray(rows)
+    np.testing.assert_allclose(_np(A).ravel()[idx], A_o.ravel()[idx], rtol=BF16_RTOL, atol=1e-6)
+    # lse_opt: the given lse_all, and lse_txt against the oracle's
+    lg = _np(lse)
+    b_i = (idx // M, idx % M)
+    for h in range(H):
+        assert np.array_equal(lg[b_i[0], h, b_i[1], 0], lse_o[b_i[0], h, b_i[1], 0].astype(np.float32))
+        np.testing.assert_allclose(lg[b_i[0], h, b_i[1], 1], lse_o[b_i[0], h, b_i[1], 1],
+                                   rtol=1e-3, atol=2e-3)
+
+
+def test_spatial_from_lse_all_matches_full_pass(av):
+    """With lse_all from the full pass's own lse output, the text-key pass
+    gives the full pass's A (weight and accumulate included)."""
+    import torch
+    from paper_2608_17995_gb300.workloads import make_transition
+    tr = make_transition("flux1024")
+    qd, kd = _dev(tr.q_img, "bf16"), _dev(tr.k_all, "bf16")
+    B, H, M, d = tr.q_img.shape
+    A1 = torch.full((B, M), 0.5, dtype=torch.float32, device="cuda")
+    lse = torch.zeros(B, H, M, 2, dtype=torch.float32, device="cuda")
+    av.avits_score_spatial(qd, kd, tr.L, tr.softmax_scale, A1, weight=0.25, accumulate=True, lse=lse)
+    A2 = torch.full((B, M), 0.5, dtype=torch.float32, device="cuda")
+    av.avits_score_spatial_lse(qd, kd[:, :, :tr.L], lse[..., 0].contiguous(), tr.softmax_scale, A2,
+                               weight=0.25, accumulate=True)
+    assert _status(av) == 0
+    np.testing.assert_allclose(_np(A2), _np(A1), rtol=2e-5, atol=1e-7)
+
+
 def _check_spatial_mask(av, orc, q, k, mask, scale, dtype, rows=None, rtol=BF16_RTOL):
     """avits_score_spatial_keymask against the masked oracle (A and the
     per-head mass through the lse pair)."""

@@ -142,3 +142,18 @@ def test_host_validation_of_the_wait_selftest(lib):
     assert f(ctypes.c_ulonglong(0), P, None) == 1
     assert f(ctypes.c_ulonglong(999), P, None) == 1
     assert f(ctypes.c_ulonglong(100000001), P, None) == 1
+
+
+def test_host_validation_of_the_lse_entry(lib):
+    """avits_score_spatial_lse: missing lse_all, L = 0 and a bad scale are
+    rejected, fp32 has no tensor-core path; nothing is launched."""
+    P = ctypes.c_void_p(16)
+    f = lib.avits_score_spatial_lse
+    args = lambda lse, dt, L, scale: (P, P, dt, 1, 2, 256, L, 64, 2 * 256 * 64, 256 * 64, 64,
+                                      2 * 32 * 64, 32 * 64, 64, lse, ctypes.c_float(scale),
+                                      ctypes.c_float(1.0), 0, P, None, P, ctypes.c_size_t(1 << 20),
+                                      None)
+    assert f(*args(None, 1, 32, 0.125)) == 1
+    assert f(*args(P, 1, 0, 0.125)) == 1
+    assert f(*args(P, 1, 32, 0.0)) == 1
+    assert f(*args(P, 0, 32, 0.125)) == 2
