@@ -250,6 +250,24 @@ def test_spatial_tc_ragged_shapes(av, orc, B, H, M, L, R, d):
     _check_spatial(av, orc, q, k, L, 1.0 / math.sqrt(d), "bf16")
 
 
+@pytest.mark.parametrize("amp,L_all", [(4.0, False), (16.0, False), (1.0, True)])
+def test_spatial_tc_large_logits_and_all_text(av, orc, amp, L_all):
+    """Logits spread far beyond the lazy running maximum's 64 log2-unit
+    window (amp 4: ~150 log2 units per row; amp 16: ~2,000, near one-hot
+    rows), so chunks keep rescuing the maximum; and every key a text key
+    (mass 1 for every row and head)."""
+    from paper_2608_17995_gb300.workloads import to_bf16_bits
+    rng = np.random.default_rng(int(amp) + 10 * L_all)
+    B, H, M, R, d = 2, 3, 300, 37, 128
+    L = M + R + 90 if L_all else 90
+    Nk = L if L_all else L + M + R
+    q = to_bf16_bits(rng.standard_normal((B, H, M, d)) * amp)
+    k = to_bf16_bits(rng.standard_normal((B, H, Nk, d)) * amp)
+    A = _check_spatial(av, orc, q, k, L, 1.0 / math.sqrt(d), "bf16")
+    if L_all:
+        np.testing.assert_allclose(A, 1.0, rtol=0, atol=1e-6)
+
+
 def test_spatial_strided_views_and_accumulate(av, orc):
     """Q as the image rows of a token-major joint [B, L+M, H, d] projection,
     K token-major too; accumulate with a weight (aggregation over blocks and
