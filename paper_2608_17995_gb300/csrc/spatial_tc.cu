@@ -41,8 +41,9 @@
 //                 come first, so the text sum is a prefix of the row sum.  At
 //                 d = 128 a 128x128 tile costs the tensor pipe and the MUFU
 //                 (32 ex2 / clock / SM) the same 512 cycles; evaluating part
-//                 of the exponentials on the FMA pipe (exp2_fma2) was measured
-//                 slower on this chip (the loop is issue-bound), so E = 0.
+//                 of the exponentials on the FMA pipe with a polynomial was
+//                 measured slower on this chip (the loop is issue-bound), so
+//                 every exponential goes to the MUFU.
 // Every wait is bounded (avits_common.cuh); on a timeout all roles stop
 // issuing, drain what they issued, release tensor memory and exit.
 #include <cuda.h>
@@ -213,25 +214,6 @@ __device__ __forceinline__ void fadd2(float& s0, float& s1, float e0, float e1) 
       : "f"(e0), "f"(e1));
 }
 
-// (d0, d1) = (a0, a1) * (b0, b1) + (c0, c1) on a packed pair.
-__device__ __forceinline__ void fma2full(float a0, float a1, float b0, float b1, float c0, float c1,
-                                         float& d0, float& d1) {
-  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
-      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
-      "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
-      : "=f"(d0), "=f"(d1)
-      : "f"(a0), "f"(a1), "f"(b0), "f"(b1), "f"(c0), "f"(c1));
-}
-
-// (p0, p1) = (p0, p1) * (r0, r1) + k on a packed pair.
-__device__ __forceinline__ void fma2v(float& p0, float& p1, float r0, float r1, float k) {
-  asm("{\n\t.reg .b64 ra, rb, rc;\n\t"
-      "mov.b64 ra, {%0, %1};\n\tmov.b64 rb, {%2, %3};\n\tmov.b64 rc, {%4, %4};\n\t"
-      "fma.rn.f32x2 ra, ra, rb, rc;\n\tmov.b64 {%0, %1}, ra;\n\t}"
-      : "+f"(p0), "+f"(p1)
-      : "f"(r0), "f"(r1), "f"(k));
-}
-
 __device__ __forceinline__ void bar_sync(int id, int count) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
@@ -249,26 +231,6 @@ __device__ __forceinline__ void merge_stat(RowStat& a, float m2, float la2, floa
   a.la = a.la * f1 + la2 * f2;
   a.lt = a.lt * f1 + lt2 * f2;
   a.m = m;
-}
-
-// 2^x on the FMA pipe for a pair of values: x clamped to [-126, 64] (a
-// clamped-high value still fails the caller's 2^64 check), j = round(x) by
-// the 1.5*2^23 addition, r = x - j in [-1/2, 1/2], 2^r by a degree-4 minimax
-// polynomial (Horner), 2^j added to the exponent field.
-__device__ __forceinline__ void exp2_fma2(float x0, float x1, float& e0, float& e1) {
-  const float kMagic = 12582912.0f;   // 1.5 * 2^23
-  x0 = fminf(fmaxf(x0, -126.0f), 64.0f);
-  x1 = fminf(fmaxf(x1, -126.0f), 64.0f);
-  float y0, y1, t0, t1, r0, r1, p0, p1;
-  ffma2(x0, x1, 1.0f, kMagic, y0, y1);          // y = x + magic (rounds x)
-  ffma2(y0, y1, 1.0f, -kMagic, t0, t1);         // t = round(x)
-  fma2full(t0, t1, -1.0f, -1.0f, x0, x1, r0, r1);   // r = x - t
-  ffma2(r0, r1, 9.570102e-03f, 5.591786e-02f, p0, p1);
-  fma2v(p0, p1, r0, r1, 2.4024744e-01f);
-  fma2v(p0, p1, r0, r1, 6.931218e-01f);
-  fma2v(p0, p1, r0, r1, 9.999993e-01f);
-  e0 = __int_as_float(__float_as_int(p0) + (__float_as_int(y0) << 23));
-  e1 = __int_as_float(__float_as_int(p1) + (__float_as_int(y1) << 23));
 }
 
 // One chunk of 16 keys that are all valid and all text (kText) or all image
@@ -310,9 +272,8 @@ __device__ __forceinline__ void process_chunk_full(const uint32_t (&r)[16], floa
   if (kText) st.lt += cs;
 }
 
-// One 16-column chunk whose first key is col0 (< Nk); the last E of its
-// exponentials (E = 0, 2 or 4) are evaluated on the FMA pipe.
-template <int E>
+// One 16-column chunk whose first key is col0 (< Nk), possibly ragged (keys
+// beyond Nk) or straddling the text / image boundary.
 __device__ __forceinline__ void process_chunk(const uint32_t (&r)[16], int col0, int Nk, int L,
                                               float c, RowStat& st) {
   float v[16];
@@ -330,15 +291,9 @@ __device__ __forceinline__ void process_chunk(const uint32_t (&r)[16], int col0,
   for (int e = 0; e < 16; e += 2) ffma2(v[e], v[e + 1], c, nm, x[e], x[e + 1]);
   float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
-  for (int e = 0; e < 16 - E; e += 4) {
+  for (int e = 0; e < 16; e += 4) {
     fadd2(s0, s1, ex2(x[e]), ex2(x[e + 1]));
-    if (e + 2 < 16 - E) fadd2(s2, s3, ex2(x[e + 2]), ex2(x[e + 3]));
-  }
-#pragma unroll
-  for (int e = 16 - E; e < 16; e += 2) {
-    float e0, e1;
-    exp2_fma2(x[e], x[e + 1], e0, e1);
-    fadd2(s2, s3, e0, e1);
+    fadd2(s2, s3, ex2(x[e + 2]), ex2(x[e + 3]));
   }
   fadd2(s0, s1, s2, s3);
   float cs = s0 + s1;
@@ -436,7 +391,7 @@ __device__ __forceinline__ void softmax_item(uint32_t tb, int c0, int Nk, int L,
   const int nch = (kKind >= kItemGeneral) ? max(0, min(4, (Nk - c0 + 15) >> 4)) : 4;
   auto chunk = [&](const uint32_t(&r)[16], int k) {
     if (kKind == kItemGeneral) {
-      if (k < nch) process_chunk<0>(r, c0 + 16 * k, Nk, L, c, st);
+      if (k < nch) process_chunk(r, c0 + 16 * k, Nk, L, c, st);
     } else if (kKind == kItemMasked) {
       const uint32_t m16 = ((k < 2 ? w0 : w1) >> (16 * (k & 1))) & 0xFFFFu;
       if (k < nch) process_chunk_masked(r, c0 + 16 * k, Nk, m16, c, st);
