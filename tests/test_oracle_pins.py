@@ -52,6 +52,13 @@ def test_spatial_matches_full_softmax(oracle_mod, seed, B, H, M, L, R, d, dt):
         np.testing.assert_allclose(np.exp(lse[..., 1] - lse[..., 0]), mass, rtol=1e-12)
     else:
         assert np.all(mass == 0) and np.all(np.isneginf(lse[..., 1]))
+    # lse over all keys (the value a model's attention forward returns, the
+    # input of the lse-based entry point) against a brute-force logsumexp
+    qf, kf = brute.as_f64(q), brute.as_f64(k)
+    logits = scale * np.einsum("bhmd,bhnd->bhmn", qf, kf)
+    mx = logits.max(-1, keepdims=True)
+    lse_ref = (mx + np.log(np.exp(logits - mx).sum(-1, keepdims=True)))[..., 0]
+    np.testing.assert_allclose(lse[..., 0], lse_ref, rtol=1e-12, atol=1e-12)
 
 
 def test_spatial_q_zero_uniform(oracle_mod):
