@@ -366,7 +366,8 @@ def run_ours(args, world, rank, local, pg):
         result["temporal_var"] = temporal_var_measure(torch, av, tr, dev, stream, peaks)
         result["spatial_keymask"] = keymask_measure(torch, av, buf, tr, sets, nsets, stream, peaks)
         result["spatial_from_lse"] = lse_measure(torch, av, buf, tr, sets, nsets, stream, peaks)
-        result["flux2048"] = flux2048_measure(torch, av, dev, stream, peaks)
+        result["flux2048"] = config_measure(torch, av, dev, stream, peaks, "flux2048")
+        result["edit"] = config_measure(torch, av, dev, stream, peaks, "edit")
     return result, tr
 
 
@@ -465,15 +466,22 @@ def warm_measure(torch, buf, sets, stream, K, per_graph=10):
             "l2": "one input set, resident in L2"}
 
 
-def flux2048_measure(torch, av, dev, stream, peaks, nsets=3):
-    """The FLUX-2048 transition (64x64 -> 128x128 tokens, M = 4096, Nk = 4608,
-    116 GFLOP in the spatial score): the whole step and the spatial call,
-    inputs rotated over nsets copies (~300 MB > L2).  At this size every CTA
-    of the spatial kernel runs ~90 items, so start-up and the finalize are a
-    small share of its time."""
+CONFIG_NOTES = {
+    "flux2048": "B=1, H=24, 64x64 -> 128x128 tokens, M=4096, L=512, Nk=4608, k=1024, nearest",
+    "edit": "B=1, H=24, 32x32 -> 64x64 tokens, M=1024, L=512, 4096 reference keys, Nk=5632, "
+            "k=205, nearest",
+}
+
+
+def config_measure(torch, av, dev, stream, peaks, name, nsets=3):
+    """Another configuration's transition: the whole step and the spatial
+    call, inputs rotated over nsets copies (> L2).  FLUX-2048 (M = 4096,
+    Nk = 4608, 116 GFLOP in the spatial score): every CTA of the spatial
+    kernel runs ~90 items, so start-up and the finalize are a small share of
+    its time.  Editing (M = 1024 with 4096 reference keys, Nk = 5632)."""
     from paper_2608_17995_gb300.pipeline import TransitionBuffers
     from paper_2608_17995_gb300.workloads import make_transition
-    t2 = make_transition("flux2048")
+    t2 = make_transition(name)
     b2 = TransitionBuffers(t2, device=dev)
     base = (b2.q, b2.k, b2.h_t, b2.h_prev, b2.latent)
     sets2 = [base] + [tuple(x.clone() for x in base) for _ in range(nsets - 1)]
@@ -495,8 +503,7 @@ def flux2048_measure(torch, av, dev, stream, peaks, nsets=3):
     return {"ms_per_step": round(ms_step, 6), "value": round(1e3 / ms_step, 1), "unit": UNIT,
             "spatial_us": round(ms_sp * 1e3, 3), "spatial_tflops": round(tf, 2),
             "spatial_frac_tensor": round(tf / peaks["bf16_tflops"], 4),
-            "status": av.avits_device_status(stream),
-            "config": "B=1, H=24, 64x64 -> 128x128 tokens, M=4096, L=512, Nk=4608, k=1024, nearest"}
+            "status": av.avits_device_status(stream), "config": CONFIG_NOTES[name]}
 
 
 def batched_schedule_measure(torch, av, dev, stream, K):
