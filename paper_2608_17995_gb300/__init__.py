@@ -9,11 +9,18 @@ fails loudly when the library has not been built (``build()``).
 
 Calls:
   avits_score_spatial       Eq. 3-5  text attention mass per image token
+                            (text_mask=: interleaved text keys)
+  avits_score_spatial_lse   Eq. 5  from the model attention's logsumexp over
+                            all keys and the text keys only
   avits_score_temporal      Sec. 3.3.2  relative step change per token
+  avits_score_spatiotemporal  both scores in one call
   avits_score_temporal_var  Eq. 6-7  step variance over N_T snapshots
   avits_fuse_select         Eq. 8-9  min-max fuse + deterministic top-k
+                            (perturb=: caller's tie-break noise)
   avits_selective_upsample  Sec. 3.2 Stage 2  packed mixed-resolution sequence
+  avits_select_upsample     selection + upsample in one launch
   avits_merge_final         Sec. 3.2 Stage 3  dense full-resolution latent
+  avits_device_status       device-side error word (read and cleared)
 """
 from __future__ import annotations
 
