@@ -35,7 +35,8 @@ __all__ = [
     "avits_score_spatial", "avits_score_spatial_workspace", "avits_score_spatial_lse",
     "avits_score_temporal",
     "avits_score_spatiotemporal",
-    "avits_score_temporal_var", "avits_fuse_select", "avits_selective_upsample",
+    "avits_score_spatial_noalloc", "avits_score_temporal_var", "avits_fuse_select",
+    "avits_selective_upsample", "avits_select_upsample",
     "avits_merge_final", "avits_merge_final_workspace", "avits_device_status",
     "avits_selftest_bounded_wait", "avits_status_string", "avits_version", "SpatialWorkspace",
 ]
