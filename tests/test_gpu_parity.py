@@ -437,7 +437,8 @@ def _run_select(av, A, V, alpha, k):
     (0, 1, 1024, 307, False, 0.5), (1, 3, 1024, 307, True, 0.5), (2, 1, 4096, 1024, True, 0.25),
     (3, 2, 640, 192, True, 1.0), (4, 1, 1, 1, False, 0.5), (5, 2, 5, 0, False, 0.5),
     (6, 1, 100, 100, True, 0.0), (7, 1, 32768, 9000, True, 0.6), (8, 4, 1000, 1, True, 0.5),
-    (9, 1, 3000, 2999, True, 0.5),
+    (9, 1, 3000, 2999, True, 0.5), (10, 2, 1600, 500, True, 0.5), (11, 1, 2048, 700, False, 0.3),
+    (12, 3, 257, 80, True, 0.5),
 ])
 def test_select_bit_exact(av, orc, seed, B, M, k, ties, alpha):
     from paper_2608_17995_gb300.workloads import random_scores
@@ -681,12 +682,16 @@ def _fused_vs_separate(av, buf, perturb=None, k=None):
 
 @pytest.mark.parametrize("name,mode", [("tiny", "nearest"), ("flux1024", "nearest"),
                                        ("flux1024", "bilinear"), ("batched", "nearest"),
-                                       ("flux2048", "nearest")])
+                                       ("flux2048", "nearest"), ("flux2048", "bilinear"),
+                                       ("edit", "nearest"), ("g40", "nearest"),
+                                       ("g40", "bilinear")])
 def test_select_upsample_fused_matches_separate(av, name, mode):
-    """One-launch selection + upsample (FLUX-2048: the two-kernel fallback)."""
+    """One-launch selection + upsample at 1, 2, 4 and 8 keys per thread
+    (M = 256, 1024, 1600, 4096), bit-identical to the two calls."""
     from paper_2608_17995_gb300.pipeline import TransitionBuffers
     from paper_2608_17995_gb300.workloads import make_transition
-    buf = TransitionBuffers(make_transition(name), mode=mode)
+    tr = make_transition("flux1024", G=40, k=480) if name == "g40" else make_transition(name)
+    buf = TransitionBuffers(tr, mode=mode)
     buf.spatial(); buf.temporal()
     _fused_vs_separate(av, buf)
 
