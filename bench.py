@@ -496,13 +496,23 @@ def config_measure(torch, av, dev, stream, peaks, name, nsets=3):
             b2.set_inputs(*sets2[s_])
             b2.spatial(stream)
 
+    def temporal():
+        for s_ in range(nsets):
+            b2.set_inputs(*sets2[s_])
+            b2.temporal(stream)
+
     ms_step = _graph_time_ms(torch, stream, step, 20) / nsets
     ms_sp = _graph_time_ms(torch, stream, spatial, 20) / nsets
+    ms_tp = _graph_time_ms(torch, stream, temporal, 20) / nsets
     flops = 2.0 * t2.B * t2.H * t2.M * t2.Nk * t2.d
     tf = flops / (ms_sp * 1e-3) / 1e12
+    tbytes = 2.0 * t2.B * t2.M * t2.D * b2.h_t.element_size() + 4.0 * t2.B * t2.M
+    tgbs = tbytes / (ms_tp * 1e-3) / 1e9
     return {"ms_per_step": round(ms_step, 6), "value": round(1e3 / ms_step, 1), "unit": UNIT,
             "spatial_us": round(ms_sp * 1e3, 3), "spatial_tflops": round(tf, 2),
             "spatial_frac_tensor": round(tf / peaks["bf16_tflops"], 4),
+            "temporal_us": round(ms_tp * 1e3, 3), "temporal_gbs": round(tgbs, 1),
+            "temporal_frac_hbm": round(tgbs / peaks["hbm_gbs"], 4),
             "status": av.avits_device_status(stream), "config": CONFIG_NOTES[name]}
 
 
