@@ -11,17 +11,26 @@
  * in spatial order (Sec. 3.2, Stage 3).  This library computes that transition:
  *
  *   avits_score_spatial       Eq. 3 + Eq. 5   per-token text attention mass
+ *     _keymask                  interleaved text keys given by a mask
+ *     _lse                      from the model attention's logsumexp
+ *     _noalloc                  without a caller workspace
  *   avits_score_temporal      Sec. 3.3.2      per-token relative step change
+ *   avits_score_spatiotemporal  both scores in one call
+ *   avits_score_temporal_var  Eq. 6-7         step variance over N_T snapshots
  *   avits_fuse_select         Sec. 3.3.3, Eq. 8 + Eq. 9   min-max, fuse, top-K
+ *     _perturbed                with caller-supplied tie-break noise (Eq. 9)
  *   avits_selective_upsample  Sec. 3.2 Stage 2   packed mixed-resolution sequence
+ *   avits_select_upsample     selection + upsample in one launch
  *   avits_merge_final         Sec. 3.2 Stage 3   dense full-resolution latent
+ *   avits_selftest_bounded_wait  test hook for the device-side failure path
  *
  * Conventions shared by every call
  * --------------------------------
  *  - Every tensor pointer is DEVICE memory owned by the caller.  The library
- *    allocates no device memory; the split-key partial sums of
+ *    allocates no device memory at run time; the split-key partial sums of
  *    avits_score_spatial and the cell map of bilinear avits_merge_final live
- *    in a caller workspace whose size a *_workspace() query returns.
+ *    in a caller workspace whose size a *_workspace() query returns (the one
+ *    exception: the static scratch array of avits_score_spatial_noalloc).
  *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
  *    stream).  Every call is asynchronous and stream ordered; none
  *    synchronises the host except avits_device_status().
