@@ -231,9 +231,9 @@ def run_ours(args, world, rank, local, pg):
     sets = [base] + [tuple(t.clone() for t in base) for _ in range(nsets - 1)]
     torch.cuda.synchronize()
 
-    # our kernels per step: spatial main + temporal (beside it) + finalize,
-    # the fused selection + upsample, the merge (bilinear: map + gather)
-    kernels_per_step = 5 if buf.mode == av.NEAREST else 6
+    # our kernels per step: spatial + temporal (beside it), the fused
+    # selection + upsample, the merge (bilinear: map + gather)
+    kernels_per_step = 4 if buf.mode == av.NEAREST else 5
     names = ["spatial", "temporal", "select", "upsample", "merge", "select_upsample"]
 
     def step(s, st):

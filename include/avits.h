@@ -101,11 +101,15 @@ typedef enum { AVITS_UP_NEAREST = 0, AVITS_UP_BILINEAR = 1 } avits_upmode;
  *         keys, the same over the text keys), natural log; -inf when a sum
  *         underflows.
  * workspace/ws_bytes : at least avits_score_spatial_workspace(...) bytes of
- *         device scratch (per-row partial statistics of the key ranges each
- *         SM handled; no initial contents are needed).  One workspace must
- *         not be used by two calls running concurrently.  The bf16
- *         tensor-core path runs two kernels (scores, then a merge launched
- *         as a programmatic dependent on the same stream).
+ *         device scratch: per-row partial statistics of the key ranges each
+ *         SM handled, ready flags and one 64-bit head-sum word per row.  It
+ *         must be ZERO-FILLED before its first use (e.g. cudaMemset); every
+ *         call that completes leaves it zero-filled again, so it is reused as
+ *         is, also by calls with other sizes.  After a call that reported
+ *         AVITS_ERR_TIMEOUT (avits_device_status), zero it again.  One
+ *         workspace must not be used by two calls running concurrently.  The
+ *         bf16 tensor-core path is one kernel; H <= 255 on that path (more
+ *         heads take the CUDA-core path).
  * ---------------------------------------------------------------------- */
 avits_status avits_score_spatial(const void* q_img, const void* k_all, avits_dtype dt,
                                  int B, int H, int M, int Nk, int L, int d,
@@ -166,11 +170,13 @@ const char* avits_score_spatial_noalloc_error(void);
  *           accumulate and A as avits_score_spatial.
  * lse_all : [B,H,M] fp32, contiguous: natural-log logsumexp of s*q_i.k_j over
  *           every key of the joint sequence, for the same s and the same
- *           queries.  Inconsistent values give masses outside [0, 1].
+ *           queries.  Each per-head mass is clamped to [0, 1] before the
+ *           head mean (inconsistent values would give masses outside it).
  * lse_opt : NULL or [B,H,M,2]: (lse_all as given, lse_txt).
- * workspace : avits_score_spatial_workspace(dt, B, H, M, L, d) bytes.
- * Tensor-core path only (bf16, d in {64,128}, 16-byte aligned layout);
- * anything else returns AVITS_ERR_UNSUPPORTED.
+ * workspace : avits_score_spatial_workspace(dt, B, H, M, L, d) bytes,
+ *           zero-filled before first use as for avits_score_spatial.
+ * Tensor-core path only (bf16, d in {64,128}, 16-byte aligned layout,
+ * H <= 255); anything else returns AVITS_ERR_UNSUPPORTED.
  * ---------------------------------------------------------------------- */
 avits_status avits_score_spatial_lse(const void* q_img, const void* k_txt, avits_dtype dt,
                                      int B, int H, int M, int L, int d, int64_t q_sb,

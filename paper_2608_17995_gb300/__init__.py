@@ -181,7 +181,9 @@ def avits_score_spatial_workspace(dtype, B, H, M, Nk, d) -> int:
 
 class SpatialWorkspace:
     """Device scratch for avits_score_spatial, grown on demand (reused by
-    calls on one stream; its contents need no initialisation)."""
+    calls on one stream).  Allocated zero-filled: the counters at its start
+    must be zero before a call, and every completed call leaves them zero;
+    after a call that reported a device timeout, call reset()."""
 
     def __init__(self, device=None):
         self.buf = None
@@ -192,7 +194,7 @@ class SpatialWorkspace:
         if nbytes == 0:
             return None, 0
         if self.buf is None or self.buf.numel() < nbytes:
-            self.buf = torch.empty(nbytes, dtype=torch.uint8, device=self.device or "cuda")
+            self.buf = torch.zeros(nbytes, dtype=torch.uint8, device=self.device or "cuda")
         return self.buf, self.buf.numel()
 
     def reset(self):

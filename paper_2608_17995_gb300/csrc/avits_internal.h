@@ -38,7 +38,12 @@ struct SpatialArgs {
 // layout is not eligible (the caller then uses the CUDA-core path).
 bool spatial_tc_eligible(const SpatialArgs& a);
 size_t spatial_tc_workspace(int B, int H, int M, int Nk, int d, int num_sms);
-// Launches issued between the main spatial kernel and its merge kernel.
+// Leading bytes of that workspace that must be zero before a call (the row
+// words and ready flags of the in-kernel merge); a completed call leaves them
+// zero again.
+size_t spatial_tc_zeroed_bytes(int B, int H, int M, int Nk, int d, int num_sms);
+// Launches issued right after the spatial kernel, as its programmatic
+// dependents (they must not complete before it does).
 using LaunchHook = std::function<cudaError_t(cudaStream_t)>;
 cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s,
                               const LaunchHook* between = nullptr);

@@ -24,7 +24,8 @@ namespace avits {
 namespace {
 
 // Upper bound of the scratch one call may use (per-row partial statistics
-// of every (SM, key range) piece).  Covers the 1024^2 and 2048^2 FLUX-shaped
+// of every (SM, key range) piece, the ready flags and the per-row head-sum
+// words).  Covers the 1024^2 and 2048^2 FLUX-shaped
 // transitions, the editing shape and a batch of 8 second transitions.
 constexpr size_t kStaticScratchBytes = 8u << 20;
 
@@ -95,7 +96,12 @@ avits_status avits_score_spatial_noalloc(const void* q_img, const void* k_all, a
     return AVITS_ERR_CUDA;
   }
   a.ws = scratch;
-  e = launch_spatial_tc(a, sms, static_cast<cudaStream_t>(stream));
+  // the row words and ready flags of the in-kernel merge start at zero; a
+  // call that stopped on a timeout may have left some set, so every call
+  // clears them (a memset on the stream: no allocation)
+  e = cudaMemsetAsync(scratch, 0, spatial_tc_zeroed_bytes(B, H, M, Nk, d, sms),
+                      static_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess) e = launch_spatial_tc(a, sms, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) {
     cudaGetLastError();
     return AVITS_ERR_CUDA;

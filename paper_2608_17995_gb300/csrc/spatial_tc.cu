@@ -12,13 +12,33 @@
 //   unit  = (b, h, 256 query rows = two 128-row tiles)
 //   item  = (unit, 128-key tile)
 // The B*H*ceil(M/256)*ceil(Nk/128) items are split into equal contiguous
-// ranges, one per CTA, so every SM issues the same number of MMA tiles.  Every
-// (CTA, unit) piece stores its per-row partial statistics (max, sum over all
-// keys, sum over text keys; the two column halves merged in shared memory)
-// in the workspace; a second,
-// small kernel (spatial_finalize_kernel, launched as a programmatic dependent
-// of the first) merges the pieces of each (row, head) in slot order and sums
-// the heads in head order, so the result does not depend on CTA timing.
+// ranges, one per CTA, so every SM issues the same number of MMA tiles.  A
+// unit whose key tiles fall into several CTAs' ranges leaves one piece of
+// per-row partial statistics (max, sum over all keys, sum over text keys;
+// the two column halves merged in shared memory) per CTA.  The merge is part
+// of this kernel:
+//   * the CTA holding the unit's first item is its merger.  That piece is the
+//     last segment of its range, so the other pieces (the first segments of
+//     the following CTAs) are mostly finished long before.  Their holders
+//     store each row's statistics as two 64-bit words, (m, l_all) and
+//     (l_txt, l_all), each written in one single-copy-atomic store; l_all
+//     is never 0 (the row's largest term is 1), so a word is either the
+//     zero left by the previous call or this call's value.  The merger
+//     polls both words of every row until they are non-zero, clears them,
+//     merges the pieces in slot order and forms the text mass of every
+//     (row, head) of the unit.  No flag and no fence stand between a piece
+//     and its merger: a piece is one store away from it;
+//   * the head mean of Eq. 3 is an exact integer sum: each (row, head) mass
+//     in [0, 1] is added as a 40-bit fixed-point number to one 64-bit word per
+//     row that also counts the heads (top byte) and the NaN masses (next
+//     byte).  The atomic add returns the new word, so the head that completes
+//     the count writes A and clears the word for the next call.  Integer
+//     addition is associative: A does not depend on the order in which CTAs
+//     finish.
+// The workspace is zero between calls: the caller zeroes it once, and a call
+// that completes clears every word it used (head-sum words and pieces), so
+// a later call with other sizes, whose row words may lie where these pieces
+// were, also finds zeros.
 //
 // Roles (19 warps):
 //   warp 0        TMA producer: Q tile 0, the first K tile, Q tile 1, then the
@@ -103,7 +123,9 @@ struct TcParams {
   int accumulate;
   float* A;
   float* lse;
-  float* part;      // [B*n_qp][H][max_parts][256][3]
+  unsigned long long* part;  // [n_units][max_parts][256][2] pieces of the non-merger CTAs
+  unsigned long long* acc;   // [B][n_qp * 256] head count | NaN count | fixed-point mass sum
+  int rows_pad;     // n_qp * 256
   unsigned int* status;
   const uint8_t* tmask;   // [B,Nk] text-key mask, or NULL (text keys = the first L)
   const float* lse_all;   // [B,H,M] caller's logsumexp over all keys (natural log), or NULL
@@ -323,6 +345,67 @@ __device__ __forceinline__ void process_chunk(const uint32_t (&r)[16], int col0,
   }
 }
 
+// ------------------------------------------------ merge across CTAs (gpu) --
+__device__ __forceinline__ unsigned long long pack2(float lo, float hi) {
+  return (unsigned long long)__float_as_uint(lo) | ((unsigned long long)__float_as_uint(hi) << 32);
+}
+__device__ __forceinline__ void st_word(unsigned long long* a, unsigned long long v) {
+  asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(a), "l"(v) : "memory");
+}
+__device__ __forceinline__ unsigned long long ld_word(const unsigned long long* a) {
+  unsigned long long v;
+  asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(v) : "l"(a) : "memory");
+  return v;
+}
+
+// Poll a piece's two words until both hold this call's values (non-zero);
+// bounded like the mbarrier waits.
+__device__ __forceinline__ bool piece_wait(const unsigned long long* w, unsigned long long& w0,
+                                           unsigned long long& w1, volatile int* abort_flag,
+                                           unsigned int* st) {
+  w0 = ld_word(w);
+  w1 = ld_word(w + 1);
+  if (w0 != 0ull && w1 != 0ull) return true;
+  const unsigned long long t0 = globaltimer_ns();
+  for (unsigned long long it = 1; it < kWaitMaxIters; ++it) {
+    if (w0 == 0ull) w0 = ld_word(w);
+    if (w1 == 0ull) w1 = ld_word(w + 1);
+    if (w0 != 0ull && w1 != 0ull) return true;
+    if ((it & 15ull) == 0) {
+      if (abort_flag && *abort_flag) return false;
+      if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+    }
+  }
+  raise_status(st, AVITS_ERR_TIMEOUT);
+  if (abort_flag) *abort_flag = 1;
+  return false;
+}
+
+// Fixed-point head sum (Eq. 3): word = heads << 56 | NaN masses << 48 | sum of
+// round(mass * 2^40).  H <= 255, so neither count overflows its byte and the
+// sum stays below 2^48.
+
+__device__ __forceinline__ void head_sum_add(const TcParams& p, int b, int row, float mass) {
+  unsigned long long inc = 1ull << 56;
+  if (mass != mass)
+    inc |= 1ull << 48;
+  else
+    inc += __float2ull_rn(fminf(fmaxf(mass, 0.f), 1.f) * 0x1p40f);
+  unsigned long long* w = p.acc + (long long)b * p.rows_pad + row;
+  const unsigned long long v = atomicAdd(w, inc) + inc;
+  if ((int)(v >> 56) != p.H) return;
+  *w = 0ull;   // every head is in: clear the word for the next call
+  float a;
+  if ((v >> 48) & 0xFFull) {
+    a = __int_as_float(0x7fc00000);
+  } else {
+    const double mean = (double)(v & ((1ull << 48) - 1ull)) * 0x1p-40 / (double)p.H;
+    a = (float)((double)p.weight * mean);
+  }
+  float* ap = p.A + (long long)b * p.M + row;
+  *ap = p.accumulate ? *ap + a : a;
+}
+
 // Kinds of the 64 keys a softmax warp reduces per item.
 enum ItemKind { kItemImage = 0, kItemText = 1, kItemGeneral = 2, kItemMasked = 3 };
 
@@ -434,10 +517,65 @@ __device__ __forceinline__ int pieces(int u, int n_kt, int per) {
   return ((u + 1) * n_kt - 1) / per - (u * n_kt) / per + 1;
 }
 
+// End of a segment, for the thread of row `rowu` of unit u holding the CTA's
+// piece st (both column halves merged).  A non-merger stores the piece; the
+// merger (slot 0) collects the other pieces, merges all of them in slot
+// order, forms the text mass (Eq. 5) and adds it to the row's head sum.
+__device__ __forceinline__ void unit_piece_done(const TcParams& p, int u, int rowu, RowStat st,
+                                                volatile int* abort_flag) {
+  const int slot = (int)blockIdx.x - first_cta(u, p.n_kt, p.per);
+  if (slot != 0) {
+    unsigned long long* w = p.part + (((long long)u * p.max_parts + slot) * kUnitRows + rowu) * 2;
+    st_word(w, pack2(st.m, st.la));
+    st_word(w + 1, pack2(st.lt, st.la));
+    return;
+  }
+  const int np = pieces(u, p.n_kt, p.per);
+  bool ok = true;
+#pragma unroll 1
+  for (int s = 1; s < np && ok; ++s) {
+    unsigned long long* w = p.part + (((long long)u * p.max_parts + s) * kUnitRows + rowu) * 2;
+    unsigned long long w0, w1;
+    ok = piece_wait(w, w0, w1, abort_flag, p.status);
+    if (!ok) break;
+    // consumed: zero, so that a completed call leaves the whole workspace
+    // zero whatever layout (shape) the next call gives it
+    st_word(w, 0ull);
+    st_word(w + 1, 0ull);
+    merge_stat(st, __uint_as_float((uint32_t)w0), __uint_as_float((uint32_t)(w0 >> 32)),
+               __uint_as_float((uint32_t)w1));
+  }
+  if (!ok) return;
+  const int bh = u / p.n_qp, qp = u - bh * p.n_qp;
+  const int b = bh / p.H, h = bh - b * p.H;
+  const int row = qp * kUnitRows + rowu;
+  if (row >= p.M) return;
+  const float ln2 = 0.69314718055994530942f;
+  float* lp = p.lse ? p.lse + (((long long)b * p.H + h) * p.M + row) * 2 : nullptr;
+  float mass;
+  if (p.lse_all) {
+    // the keys of this pass are the text keys only: mass = exp(lse_txt -
+    // lse_all) against the caller's logsumexp over all keys
+    const float la_all = p.lse_all[((long long)b * p.H + h) * p.M + row];
+    mass = st.lt > 0.f ? exp2f(st.m + log2f(st.lt) - la_all * 1.4426950408889634f) : 0.f;
+    if (lp) {
+      lp[0] = la_all;
+      lp[1] = st.lt > 0.f ? (st.m + log2f(st.lt)) * ln2 : -INFINITY;
+    }
+  } else {
+    mass = st.lt / st.la;
+    if (lp) {
+      lp[0] = (st.m + __log2f(st.la)) * ln2;
+      lp[1] = st.lt > 0.f ? (st.m + __log2f(st.lt)) * ln2 : -INFINITY;
+    }
+  }
+  head_sum_add(p, b, row, mass);
+}
+
 // kMask: the text keys come from the caller's key mask (p.tmask) instead of
 // being the first L; a separate instance keeps the plain kernel unchanged.
 template <int D, bool kMask>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __maxnreg__(88)
 spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                   const TcParams p) {
   using C = Cfg<D>;
@@ -491,8 +629,9 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
   tc_fence_after();
   const uint32_t tmem = bars->tmem_base;
   volatile int* abort_flag = &bars->abort;
-  // the merge kernel may be scheduled now (it waits for this grid to
-  // finish); a softmax thread signals it, keeping the producer free
+  // the next kernel may be scheduled now (it waits for this grid to finish
+  // before it reads anything); a softmax thread signals it, keeping the
+  // producer free
   if (threadIdx.x == 64) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (warp == 0) {
@@ -670,8 +809,8 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
       }
       // the two column halves of this tile's rows meet in shared memory
       // (a buffer per segment parity, so one barrier per segment suffices);
-      // half 0 merges them and stores the CTA's piece of the unit, slot
-      // CTA - first CTA of u, which halves what the finalize kernel loads
+      // half 0 merges them into the CTA's piece of the unit and takes it
+      // through the merge across CTAs
       float* xs = xch + (((sgi & 1) * kQTiles + t) * kBM + rowt) * 3;
       if (half == 1) {
         xs[0] = st.m;
@@ -684,12 +823,7 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
         bar_sync(2, 8 * 32);
       if (half == 0) {
         merge_stat(st, xs[0], xs[1], xs[2]);
-        const int u = seg.u;
-        const int slot = (int)blockIdx.x - first_cta(u, p.n_kt, p.per);
-        float* pp = p.part + (((long long)u * p.max_parts + slot) * kUnitRows + rowu) * 3;
-        pp[0] = st.m;
-        pp[1] = st.la;
-        pp[2] = st.lt;
+        unit_piece_done(p, seg.u, rowu, st, abort_flag);
       }
       ++sgi;
       li0 += seg.nk;
@@ -703,87 +837,6 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                  "r"(kTmemCols));
-  }
-}
-
-// Second kernel: merge the pieces of every (row, head) in slot order, then the
-// head mean of Eq. 3.  Block = 32 rows x 32 head lanes; thread (r, hl) merges
-// heads hl, hl+32, ... of row r (all loads of a head issued before its
-// merge), then thread (r, 0) adds the per-head masses in head order from
-// shared memory.  Launched as a programmatic dependent of spatial_tc_kernel:
-// it waits for the producer grid to complete before reading the pieces.
-constexpr int kFinRows = 32, kFinHeads = 32;
-
-__global__ void __launch_bounds__(kFinRows * kFinHeads)
-spatial_finalize_kernel(const TcParams p) {
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-  // the main grid has completed: the next kernel may start its prologue
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  __shared__ float mass_s[kFinHeads][kFinRows + 1];
-  const int r = threadIdx.x % kFinRows, hl = threadIdx.x / kFinRows;
-  const int row_g = blockIdx.x * kFinRows + r;            // over B * n_qp * 256
-  const int rows_per_b = p.n_qp * kUnitRows;
-  const int b = row_g / rows_per_b;
-  const int row = row_g - b * rows_per_b;                  // row within the element
-  const int qp = row / kUnitRows, rowu = row - qp * kUnitRows;
-  const float ln2 = 0.69314718055994530942f;
-  float sum = 0.f;   // this thread's heads, in head order
-  if (b < p.B) {
-    for (int h = hl; h < p.H; h += kFinHeads) {
-      const int u = (b * p.H + h) * p.n_qp + qp;
-      const int np = pieces(u, p.n_kt, p.per);
-      const float* q = p.part + ((long long)u * p.max_parts * kUnitRows + rowu) * 3;
-      RowStat acc{-INFINITY, 0.f, 0.f};
-      for (int s0 = 0; s0 < np; s0 += 6) {
-        float v[6][3];
-#pragma unroll
-        for (int k = 0; k < 6; ++k)
-          if (s0 + k < np) {
-            const float* qs = q + (long long)(s0 + k) * kUnitRows * 3;
-            v[k][0] = __ldcg(qs);
-            v[k][1] = __ldcg(qs + 1);
-            v[k][2] = __ldcg(qs + 2);
-          }
-#pragma unroll
-        for (int k = 0; k < 6; ++k)
-          if (s0 + k < np) merge_stat(acc, v[k][0], v[k][1], v[k][2]);
-      }
-      if (p.lse_all) {
-        // the keys of this pass are the text keys only: mass = exp(lse_txt -
-        // lse_all) against the caller's logsumexp over all keys
-        float ratio = 0.f;
-        if (row < p.M) {
-          const float la_all = p.lse_all[((long long)b * p.H + h) * p.M + row];
-          ratio = acc.lt > 0.f ? exp2f(acc.m + log2f(acc.lt) - la_all * 1.4426950408889634f)
-                               : 0.f;
-          if (p.lse) {
-            float* lp = p.lse + (((long long)b * p.H + h) * p.M + row) * 2;
-            lp[0] = la_all;
-            lp[1] = acc.lt > 0.f ? (acc.m + log2f(acc.lt)) * ln2 : -INFINITY;
-          }
-        }
-        sum += ratio;
-      } else {
-        sum += acc.lt / acc.la;
-        if (p.lse && row < p.M) {
-          float* lp = p.lse + (((long long)b * p.H + h) * p.M + row) * 2;
-          lp[0] = (acc.m + __log2f(acc.la)) * ln2;
-          lp[1] = acc.lt > 0.f ? (acc.m + __log2f(acc.lt)) * ln2 : -INFINITY;
-        }
-      }
-    }
-  }
-  mass_s[hl][r] = sum;
-  __syncthreads();
-  if (hl == 0 && b < p.B && row < p.M) {
-    // heads 0..31 first-round partials are in head order; for H > 32 each
-    // lane's partial already holds its heads hl, hl+32, ... in order
-    float tot = 0.f;
-    const int lanes = p.H < kFinHeads ? p.H : kFinHeads;
-    for (int k = 0; k < lanes; ++k) tot += mass_s[k][r];
-    const float a = p.weight * (tot / (float)p.H);
-    float* ap = p.A + (long long)b * p.M + row;
-    *ap = p.accumulate ? *ap + a : a;
   }
 }
 
@@ -831,7 +884,7 @@ bool make_map(CUtensorMap* map, const void* base, int B, int H, int rows, int d,
 struct Plan {
   int n_qp, n_kt, n_units, max_parts, grid;
   long long total, per;
-  size_t bytes;
+  size_t acc_bytes, part_bytes, bytes;
 };
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
@@ -847,7 +900,10 @@ Plan make_plan(int B, int H, int M, int Nk, int num_sms) {
   if (pl.per < 1) pl.per = 1;
   pl.grid = (int)((pl.total + pl.per - 1) / pl.per);
   pl.max_parts = (int)((pl.n_kt + pl.per - 1) / pl.per) + 1;
-  pl.bytes = align256(sizeof(float) * 3 * (size_t)pl.n_units * pl.max_parts * kUnitRows);
+  // [head-sum words][pieces: two words per row], all zero between calls
+  pl.acc_bytes = align256(sizeof(unsigned long long) * (size_t)B * pl.n_qp * kUnitRows);
+  pl.part_bytes = align256(2 * sizeof(unsigned long long) * (size_t)pl.n_units * pl.max_parts * kUnitRows);
+  pl.bytes = pl.acc_bytes + pl.part_bytes;
   return pl;
 }
 
@@ -882,9 +938,6 @@ cudaError_t set_smem_once() {
   if (e == cudaSuccess) e = smem_attrs<spatial_tc_kernel<128, true>, 128>();
   if (e == cudaSuccess) e = smem_attrs<spatial_tc_kernel<64, false>, 64>();
   if (e == cudaSuccess) e = smem_attrs<spatial_tc_kernel<64, true>, 64>();
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(spatial_finalize_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
-                             cudaSharedmemCarveoutMaxShared);
   if (e == cudaSuccess && dev >= 0 && dev < 64) __atomic_store_n(&done[dev], 1, __ATOMIC_RELEASE);
   return e;
 }
@@ -898,12 +951,18 @@ bool spatial_tc_eligible(const SpatialArgs& a) {
   if (!strides_ok(a.B, a.H, a.q_sb, a.q_sh, a.q_sn)) return false;
   if (!strides_ok(a.B, a.H, a.k_sb, a.k_sh, a.k_sn)) return false;
   if (!(a.scale > 0.f)) return false;
+  if (a.H > 255) return false;   // the head count of the fixed-point head sum is one byte
   const long long n_qp = (a.M + kUnitRows - 1) / kUnitRows, n_kt = (a.Nk + kBN - 1) / kBN;
   if ((long long)a.B * a.H * n_qp * (n_kt + 1) >= (1ll << 31)) return false;
   return encode_fn() != nullptr;
 }
 
 size_t spatial_tc_workspace(int B, int H, int M, int Nk, int d, int num_sms) {
+  (void)d;
+  return make_plan(B, H, M, Nk, num_sms).bytes;
+}
+
+size_t spatial_tc_zeroed_bytes(int B, int H, int M, int Nk, int d, int num_sms) {
   (void)d;
   return make_plan(B, H, M, Nk, num_sms).bytes;
 }
@@ -925,7 +984,9 @@ cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s,
   p.accumulate = a.accumulate;
   p.A = a.A;
   p.lse = a.lse;
-  p.part = reinterpret_cast<float*>(ws);
+  p.acc = reinterpret_cast<unsigned long long*>(ws);
+  p.part = reinterpret_cast<unsigned long long*>(ws + pl.acc_bytes);
+  p.rows_pad = pl.n_qp * kUnitRows;
   p.status = a.status;
   p.tmask = a.tmask;
   p.lse_all = a.lse_all;
@@ -947,20 +1008,7 @@ cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s,
     e = (*between)(s);
     if (e != cudaSuccess) return e;
   }
-  // the merge runs as a programmatic dependent: it may be scheduled while the
-  // main kernel drains and waits (griddepcontrol.wait) for its completion
-  cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3((unsigned)((a.B * pl.n_qp * kUnitRows + kFinRows - 1) / kFinRows));
-  cfg.blockDim = dim3(kFinRows * kFinHeads);
-  cfg.dynamicSmemBytes = 0;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, spatial_finalize_kernel, p);
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 }  // namespace avits
