@@ -618,6 +618,24 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
   // Q and K may come from the kernel before this one on the stream; tensor
   // memory is only taken once that kernel has finished
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  if (threadIdx.x == 0) {
+    // the first segment's Q tiles and first K tile go out before tensor
+    // memory is taken (the copies only need the barriers initialised above);
+    // the producer loop below skips them
+    const Segment seg = segment_at(it_begin, it_end, p.n_kt);
+    const int bh = seg.u / p.n_qp, qp = seg.u - bh * p.n_qp;
+    const int b = bh / p.H, h = bh - b * p.H;
+    mbar_arrive_expect_tx(&bars->q_full[0], C::kTileBytes);
+    for (int cb = 0; cb < C::kCB; ++cb)
+      tma_load_4d(sQ + cb * (kBM * 128), &tmQ, cb * 64, qp * kUnitRows, h, b, &bars->q_full[0]);
+    mbar_arrive_expect_tx(&bars->k_full[0], C::kTileBytes);
+    for (int cb = 0; cb < C::kCB; ++cb)
+      tma_load_4d(sK + cb * (kBM * 128), &tmK, cb * 64, seg.kt0 * kBN, h, b, &bars->k_full[0]);
+    mbar_arrive_expect_tx(&bars->q_full[1], C::kTileBytes);
+    for (int cb = 0; cb < C::kCB; ++cb)
+      tma_load_4d(sQ + C::kTileBytes + cb * (kBM * 128), &tmQ, cb * 64, qp * kUnitRows + kBM, h,
+                  b, &bars->q_full[1]);
+  }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_u32(&bars->tmem_base)),
@@ -649,11 +667,12 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
         // MMAs of the previous one
         if (sg > 0) ok = mbar_wait_bounded(&bars->q_empty, (uint32_t)((sg & 1) ^ 1), abort_flag, p.status);
         if (!ok) break;
+        const bool first = (sg == 0);   // Q tiles and K tile 0 already issued
         ++sg;   // Q of this segment is being issued
-        q_armed = 0;
+        q_armed = first ? kQTiles : 0;
         for (int j = 0; j < seg.nk; ++j, ++li) {
           // Q tile 0 before the first K tile, Q tile 1 right after it
-          if (j == 0 || (j == 1 && kQTiles > 1)) {
+          if (!first && (j == 0 || (j == 1 && kQTiles > 1))) {
             const int t = j;
             ++q_armed;
             mbar_arrive_expect_tx(&bars->q_full[t], C::kTileBytes);
@@ -668,6 +687,7 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
             ok = mbar_wait_bounded(&bars->k_full[0], 0, abort_flag, p.status);
             if (!ok) break;
           }
+          if (li == 0) continue;   // K tile 0 went out before the set-up
           const int stage = (int)(li % C::kStages);
           const uint32_t ph = (uint32_t)((li / C::kStages) & 1);
           ok = mbar_wait_bounded(&bars->k_empty[stage], ph ^ 1u, abort_flag, p.status);
@@ -677,7 +697,7 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
             tma_load_4d(sK + stage * C::kTileBytes + cb * (kBM * 128), &tmK, cb * 64,
                         (seg.kt0 + j) * kBN, h, b, &bars->k_full[stage]);
         }
-        if (ok && seg.nk == 1) {   // a one-tile segment still needs Q tile 1
+        if (ok && seg.nk == 1 && !first) {   // a one-tile segment still needs Q tile 1
           ++q_armed;
           mbar_arrive_expect_tx(&bars->q_full[1], C::kTileBytes);
           for (int cb = 0; cb < C::kCB; ++cb)
