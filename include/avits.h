@@ -138,11 +138,19 @@ size_t avits_score_spatial_workspace(avits_dtype dt, int B, int H, int M, int Nk
  * GPU that loads the library until the process exits.  A call whose shapes
  * need more returns AVITS_ERR_INVALID_ARG before launching anything, with the
  * sizes in avits_score_spatial_noalloc_error().  The call allocates nothing.
+ *  - The scratch a shape needs grows with the device's SM count (per-row
+ *    statistics are kept per SM and key range): on a 152-SM GB300 the
+ *    FLUX-1024 shape needs 1.2 MB and the batched second transition
+ *    (B = 8, H = 24, M = 640, Nk = 1152) 4.8 MB, so a shape that fits on one
+ *    GPU may be refused on a part with more SMs.
  *  - The first call on each device looks up the array's device address;
- *    make that first call before any stream capture on that device.
+ *    make that first call before any stream capture on that device (a
+ *    first call during a capture is refused, the reason in
+ *    avits_score_spatial_noalloc_error()).
  *  - All calls on a device share the one array: calls that may overlap on
  *    the GPU (other streams, other host threads) race and must be ordered
- *    by the caller.  Nothing in the array needs clearing between calls.
+ *    by the caller.  Each call clears, on its stream, the part of the array
+ *    it uses before its kernel runs, so nothing needs clearing by the caller.
  * ---------------------------------------------------------------------- */
 avits_status avits_score_spatial_noalloc(const void* q_img, const void* k_all, avits_dtype dt,
                                          int B, int H, int M, int Nk, int L, int d,
@@ -155,7 +163,7 @@ avits_status avits_score_spatial_noalloc(const void* q_img, const void* k_all, a
 size_t avits_score_spatial_noalloc_limit(void);
 
 /* Why the last avits_score_spatial_noalloc call on this thread was refused
- * for its size ("" otherwise). */
+ * (its size, or a first call made during a stream capture; "" otherwise). */
 const char* avits_score_spatial_noalloc_error(void);
 
 /* ------------------------------------------------------------------------
@@ -341,8 +349,9 @@ avits_status avits_select_upsample(const float* A, const float* V, const float* 
  * Final merge, Sec. 3.2 Stage 3: expand every remaining token to full
  * resolution and lay the tokens out in spatial (raster) order.
  * A token at (y,x) with span s covers cells [y,y+s) x [x,x+s) of the
- * full_h x full_w frame; the tokens must tile the frame exactly once
- * (otherwise AVITS_ERR_COVERAGE is raised on the device).
+ * full_h x full_w frame; the tokens must tile the frame exactly once:
+ * a cell covered twice, a cell left uncovered and a token outside the frame
+ * each raise AVITS_ERR_COVERAGE on the device, in both modes.
  *   nearest  : full-res pixel (Y,X) takes token pixel ((Y-2y)/s, (X-2x)/s).
  *   bilinear : only for spans {1,2} (one transition): span-1 tokens are
  *              copied; the low-res grid is rebuilt (span-2 tokens as they are,
@@ -350,7 +359,10 @@ avits_status avits_select_upsample(const float* A, const float* V, const float* 
  *              span-2 cells take its half-pixel-centred 2x bilinear resize.
  * mixed : [B,N,C*4].  pos [B,N,2], span [B,N] int32.
  * out_full : [B,full_h*full_w,C*4] same dtype.
- * workspace : avits_merge_final_workspace() bytes (0 for nearest).
+ * workspace : avits_merge_final_workspace() bytes (both modes), 16-byte
+ *             aligned, ZERO-FILLED before its first use; the calls keep it
+ *             consistent afterwards (nearest: a claim map tagged per call and
+ *             a counter each call clears; bilinear: a cell map it refills).
  * ---------------------------------------------------------------------- */
 avits_status avits_merge_final(const void* mixed, avits_dtype dt, int B, int N,
                                const int32_t* pos, const int32_t* span, int full_h, int full_w,

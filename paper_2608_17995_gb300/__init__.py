@@ -35,7 +35,8 @@ __all__ = [
     "avits_score_spatial", "avits_score_spatial_workspace", "avits_score_spatial_lse",
     "avits_score_temporal",
     "avits_score_spatiotemporal",
-    "avits_score_spatial_noalloc", "avits_score_temporal_var", "avits_fuse_select",
+    "avits_score_spatial_noalloc", "avits_score_spatial_noalloc_limit",
+    "avits_score_temporal_var", "avits_fuse_select",
     "avits_selective_upsample", "avits_select_upsample",
     "avits_merge_final", "avits_merge_final_workspace", "avits_device_status",
     "avits_selftest_bounded_wait", "avits_status_string", "avits_version", "SpatialWorkspace",
@@ -96,6 +97,10 @@ def lib():
                                   i32, i32, i32, i32, vp, vp, i32, vp, vp, vp, vp, vp, vp],
         "avits_merge_final": [vp, i32, i32, i32, vp, vp, i32, i32, i32, i32, i32, vp, vp, sz, vp],
         "avits_merge_final_workspace": [i32, i32, i32, i32],
+        "avits_score_spatial_noalloc": [vp, vp, i32, i32, i32, i32, i32, i32, i32, i64, i64, i64,
+                                        i64, i64, i64, f32, f32, i32, vp, vp, vp],
+        "avits_score_spatial_noalloc_limit": [],
+        "avits_score_spatial_noalloc_error": [],
         "avits_device_status": [vp],
         "avits_selftest_bounded_wait": [ctypes.c_ulonglong, vp, vp],
         "avits_status_string": [i32],
@@ -106,9 +111,11 @@ def lib():
         fn = getattr(L, name)
         fn.argtypes = args
         fn.restype = ctypes.c_int
-    for name in ("avits_score_spatial_workspace", "avits_merge_final_workspace"):
+    for name in ("avits_score_spatial_workspace", "avits_merge_final_workspace",
+                 "avits_score_spatial_noalloc_limit"):
         getattr(L, name).restype = ctypes.c_size_t
-    for name in ("avits_status_string", "avits_last_error_string", "avits_version"):
+    for name in ("avits_status_string", "avits_last_error_string", "avits_version",
+                 "avits_score_spatial_noalloc_error"):
         getattr(L, name).restype = ctypes.c_char_p
     _lib = L
     return L
@@ -404,13 +411,6 @@ def avits_score_spatial_noalloc(q_img, k_all, L: int, softmax_scale: float, A, w
     bf16 tensor-core shapes only.  Calls on one device must not overlap."""
     L_ = lib()
     fn = L_.avits_score_spatial_noalloc
-    if fn.restype is not ctypes.c_int or not fn.argtypes:
-        vp, i32, i64, f32 = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float
-        fn.argtypes = [vp, vp, i32, i32, i32, i32, i32, i32, i32, i64, i64, i64, i64, i64, i64,
-                       f32, f32, i32, vp, vp, vp]
-        fn.restype = ctypes.c_int
-        L_.avits_score_spatial_noalloc_error.restype = ctypes.c_char_p
-        L_.avits_score_spatial_noalloc_limit.restype = ctypes.c_size_t
     B, H, M, d = q_img.shape
     Nk = k_all.shape[2]
     rc = fn(_ptr(q_img), _ptr(k_all), _dtype_code(q_img), B, H, M, Nk, L, d,
@@ -419,6 +419,12 @@ def avits_score_spatial_noalloc(q_img, k_all, L: int, softmax_scale: float, A, w
             float(softmax_scale), float(weight), 1 if accumulate else 0,
             _ptr(A), _ptr(lse), _stream(stream))
     if rc != 0:
+        err = L_.avits_score_spatial_noalloc_error()
         raise AvitsError("avits_score_spatial_noalloc", rc,
-                         L_.avits_score_spatial_noalloc_error().decode())
+                         err.decode() if isinstance(err, bytes) else "")
     return A
+
+
+def avits_score_spatial_noalloc_limit() -> int:
+    """Bytes of the fixed scratch array behind avits_score_spatial_noalloc."""
+    return int(lib().avits_score_spatial_noalloc_limit())

@@ -21,6 +21,10 @@ LIB = os.path.join(OUT_DIR, "libavits.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2", "--expt-relaxed-constexpr",
          "-I" + INCLUDE, "-I" + CSRC]
+# AVITS_NVTX=1: NVTX ranges around the C entry points (see avits_internal.h);
+# rebuild with force=True after changing it
+if os.environ.get("AVITS_NVTX") == "1":
+    FLAGS.append("-DAVITS_NVTX")
 
 
 def nvcc() -> str:

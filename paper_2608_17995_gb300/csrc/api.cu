@@ -90,6 +90,7 @@ avits_status avits_score_spatial(const void* q_img, const void* k_all, avits_dty
                                  int64_t q_sn, int64_t k_sb, int64_t k_sh, int64_t k_sn,
                                  float softmax_scale, float weight, int accumulate, float* A,
                                  float* lse_opt, void* workspace, size_t ws_bytes, void* stream) {
+  AVITS_RANGE();
   if (!q_img || !k_all || !A || !valid_dtype(dt)) return AVITS_ERR_INVALID_ARG;
   if (B <= 0 || H <= 0 || M <= 0 || Nk <= 0 || d <= 0 || L < 0 || L > Nk || Nk < M)
     return AVITS_ERR_INVALID_ARG;
@@ -116,6 +117,7 @@ avits_status avits_score_spatial_lse(const void* q_img, const void* k_txt, avits
                                      const float* lse_all, float softmax_scale, float weight,
                                      int accumulate, float* A, float* lse_opt, void* workspace,
                                      size_t ws_bytes, void* stream) {
+  AVITS_RANGE();
   if (!q_img || !k_txt || !lse_all || !A || !valid_dtype(dt)) return AVITS_ERR_INVALID_ARG;
   if (B <= 0 || H <= 0 || M <= 0 || L <= 0 || d <= 0) return AVITS_ERR_INVALID_ARG;
   if (!(softmax_scale > 0.f) || !(softmax_scale < 3.0e38f)) return AVITS_ERR_INVALID_ARG;
@@ -139,6 +141,7 @@ avits_status avits_score_spatial_keymask(const void* q_img, const void* k_all, a
                                          float softmax_scale, float weight, int accumulate,
                                          float* A, float* lse_opt, void* workspace,
                                          size_t ws_bytes, void* stream) {
+  AVITS_RANGE();
   if (!q_img || !k_all || !A || !text_mask || !valid_dtype(dt)) return AVITS_ERR_INVALID_ARG;
   if (B <= 0 || H <= 0 || M <= 0 || Nk <= 0 || d <= 0 || Nk < M) return AVITS_ERR_INVALID_ARG;
   if (!(softmax_scale > 0.f) || !(softmax_scale < 3.0e38f)) return AVITS_ERR_INVALID_ARG;
@@ -160,6 +163,7 @@ avits_status avits_score_spatial_keymask(const void* q_img, const void* k_all, a
 
 avits_status avits_score_temporal(const void* h_t, const void* h_prev, avits_dtype dt, int B,
                                   int N, int D, float eps, float* V, void* stream) {
+  AVITS_RANGE();
   if (!h_t || !h_prev || !V || !valid_dtype(dt)) return AVITS_ERR_INVALID_ARG;
   if (B <= 0 || N <= 0 || D <= 0 || !(eps >= 0.f)) return AVITS_ERR_INVALID_ARG;
   return cuda_status(launch_temporal(h_t, h_prev, dt, B, N, D, eps, V, num_sms_current(),
@@ -173,6 +177,7 @@ avits_status avits_score_spatiotemporal(const void* q_img, const void* k_all, av
                                         int accumulate, float* A, float* lse_opt, void* workspace,
                                         size_t ws_bytes, const void* h_t, const void* h_prev,
                                         int D, float eps, float* V, void* stream) {
+  AVITS_RANGE();
   if (!q_img || !k_all || !A || !h_t || !h_prev || !V || !valid_dtype(dt))
     return AVITS_ERR_INVALID_ARG;
   if (B <= 0 || H <= 0 || M <= 0 || Nk <= 0 || d <= 0 || L < 0 || L > Nk || Nk < M || D <= 0)
@@ -203,6 +208,7 @@ avits_status avits_score_spatiotemporal(const void* q_img, const void* k_all, av
 
 avits_status avits_score_temporal_var(const void* const* snaps, int n_t, avits_dtype dt, int B,
                                       int N, int D, float* V, void* stream) {
+  AVITS_RANGE();
   if (!snaps || !V || !valid_dtype(dt)) return AVITS_ERR_INVALID_ARG;
   if (n_t < 2 || n_t > kMaxSnapshots || B <= 0 || N <= 0 || D <= 0) return AVITS_ERR_INVALID_ARG;
   for (int i = 0; i < n_t; ++i)
@@ -214,6 +220,7 @@ avits_status avits_score_temporal_var(const void* const* snaps, int n_t, avits_d
 avits_status avits_fuse_select(const float* A, const float* V, int B, int M, float alpha,
                                float eps_norm, int k, float* S_opt, int32_t* sel_idx,
                                uint8_t* sel_mask_opt, int32_t* tok_offset, void* stream) {
+  AVITS_RANGE();
   return avits_fuse_select_perturbed(A, V, nullptr, B, M, alpha, eps_norm, k, S_opt, sel_idx,
                                      sel_mask_opt, tok_offset, stream);
 }
@@ -222,6 +229,7 @@ avits_status avits_fuse_select_perturbed(const float* A, const float* V, const f
                                          int B, int M, float alpha, float eps_norm, int k,
                                          float* S_opt, int32_t* sel_idx, uint8_t* sel_mask_opt,
                                          int32_t* tok_offset, void* stream) {
+  AVITS_RANGE();
   if (!A || !V || !tok_offset || (k > 0 && !sel_idx)) return AVITS_ERR_INVALID_ARG;
   if (B <= 0 || M <= 0 || M > kSelectMaxM || k < 0 || k > M) return AVITS_ERR_INVALID_ARG;
   if (!(alpha >= 0.f && alpha <= 1.f) || !(eps_norm >= 0.f)) return AVITS_ERR_INVALID_ARG;
@@ -237,6 +245,7 @@ avits_status avits_selective_upsample(const void* latent, avits_dtype dt, int B,
                                       avits_upmode mode, void* out_latent, int32_t* out_pos,
                                       int32_t* out_span, int32_t* out_src_tok,
                                       int8_t* out_src_sub, void* stream) {
+  AVITS_RANGE();
   if (!latent || !sel_mask || !tok_offset || !out_latent || !out_pos || !out_span ||
       !out_src_tok || !out_src_sub || !valid_dtype(dt))
     return AVITS_ERR_INVALID_ARG;
@@ -262,6 +271,7 @@ avits_status avits_select_upsample(const float* A, const float* V, const float* 
                                    const int32_t* span_in_opt, avits_upmode mode,
                                    void* out_latent, int32_t* out_pos, int32_t* out_span,
                                    int32_t* out_src_tok, int8_t* out_src_sub, void* stream) {
+  AVITS_RANGE();
   if (!A || !V || !tok_offset || !sel_mask || (k > 0 && !sel_idx)) return AVITS_ERR_INVALID_ARG;
   if (B <= 0 || M <= 0 || M > kSelectMaxM || k < 0 || k > M) return AVITS_ERR_INVALID_ARG;
   if (!(alpha >= 0.f && alpha <= 1.f) || !(eps_norm >= 0.f)) return AVITS_ERR_INVALID_ARG;
@@ -282,30 +292,33 @@ avits_status avits_select_upsample(const float* A, const float* V, const float* 
 }
 
 size_t avits_merge_final_workspace(avits_upmode mode, int B, int full_h, int full_w) {
-  if (mode != AVITS_UP_BILINEAR || B <= 0 || full_h <= 0 || full_w <= 0) return 0;
-  return sizeof(int32_t) * (size_t)B * full_h * full_w;
+  if ((mode != AVITS_UP_NEAREST && mode != AVITS_UP_BILINEAR) || B <= 0 || full_h <= 0 ||
+      full_w <= 0)
+    return 0;
+  return merge_workspace_bytes(B, full_h, full_w);
 }
 
 avits_status avits_merge_final(const void* mixed, avits_dtype dt, int B, int N, const int32_t* pos,
                                const int32_t* span, int full_h, int full_w, int C, int p,
                                avits_upmode mode, void* out_full, void* workspace,
                                size_t ws_bytes, void* stream) {
+  AVITS_RANGE();
   if (!mixed || !pos || !span || !out_full || !valid_dtype(dt)) return AVITS_ERR_INVALID_ARG;
   if (B <= 0 || N <= 0 || full_h <= 0 || full_w <= 0 || C <= 0) return AVITS_ERR_INVALID_ARG;
   if (p != 2) return AVITS_ERR_UNSUPPORTED;
   if (mode != AVITS_UP_NEAREST && mode != AVITS_UP_BILINEAR) return AVITS_ERR_INVALID_ARG;
   if (!aligned16(mixed) || !aligned16(out_full)) return AVITS_ERR_INVALID_ARG;
-  if (mode == AVITS_UP_BILINEAR) {
-    if ((full_h & 1) || (full_w & 1)) return AVITS_ERR_INVALID_ARG;
-    if (!workspace || ws_bytes < avits_merge_final_workspace(mode, B, full_h, full_w))
-      return AVITS_ERR_INVALID_ARG;
-  }
+  if (mode == AVITS_UP_BILINEAR && ((full_h & 1) || (full_w & 1))) return AVITS_ERR_INVALID_ARG;
+  if (!workspace || !aligned16(workspace) ||
+      ws_bytes < avits_merge_final_workspace(mode, B, full_h, full_w))
+    return AVITS_ERR_INVALID_ARG;
   return cuda_status(launch_merge(mixed, dt, B, N, pos, span, full_h, full_w, C, mode, out_full,
                                   workspace, status_word(), static_cast<cudaStream_t>(stream)));
 }
 
 avits_status avits_selftest_bounded_wait(unsigned long long limit_ns, long long* result,
                                          void* stream) {
+  AVITS_RANGE();
   if (!result || limit_ns < 1000ull || limit_ns > 100ull * 1000ull * 1000ull)
     return AVITS_ERR_INVALID_ARG;
   return cuda_status(launch_wait_selftest(limit_ns, result, status_word(),
@@ -313,6 +326,7 @@ avits_status avits_selftest_bounded_wait(unsigned long long limit_ns, long long*
 }
 
 avits_status avits_device_status(void* stream) {
+  AVITS_RANGE();
   cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_status(e);
   unsigned int w = 0, zero = 0;

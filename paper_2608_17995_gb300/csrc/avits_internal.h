@@ -8,6 +8,25 @@
 
 #include "avits.h"
 
+// NVTX ranges around the C entry points, for timeline tools: compiled in
+// with -DAVITS_NVTX (build with AVITS_NVTX=1 in the environment), nothing
+// otherwise.  NVTX v3 is header-only; without a tool attached a range costs a
+// null check.
+#ifdef AVITS_NVTX
+#include <nvtx3/nvToolsExt.h>
+namespace avits {
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+}  // namespace avits
+#define AVITS_RANGE() ::avits::NvtxRange avits_nvtx_range_(__func__)
+#else
+#define AVITS_RANGE() ((void)0)
+#endif
+
 namespace avits {
 
 // Device address of the status word of the current device (api.cu).
@@ -91,6 +110,8 @@ cudaError_t launch_upsample(const void* latent, avits_dtype dt, int B, int M, in
                             int32_t* out_src_tok, int8_t* out_src_sub, cudaStream_t s);
 
 // ---- final merge (Stage 3) --------------------------------------------------
+// Workspace of either mode: a 16-byte header and one 32-bit word per cell.
+size_t merge_workspace_bytes(int B, int fh, int fw);
 cudaError_t launch_merge(const void* mixed, avits_dtype dt, int B, int N, const int32_t* pos,
                          const int32_t* span, int fh, int fw, int C, avits_upmode mode,
                          void* out, void* ws, unsigned int* status, cudaStream_t s);

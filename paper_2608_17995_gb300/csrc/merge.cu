@@ -4,6 +4,13 @@
 //
 // Nearest: one warp per mixed token scatters its s x s cells; full-res pixel
 // (Y,X) of a token at (y,x) with span s takes token pixel ((Y-2y)/s, (X-2x)/s).
+// Coverage is checked in the same kernel: every cell is claimed by an
+// atomicExch of this call's tag into a claim map in the caller's workspace
+// (an old value equal to the tag = a cell covered twice), and every CTA adds
+// (1 << 40) | cells claimed to one 64-bit word; the CTA whose add completes
+// the CTA count compares the claimed total with B * fh * fw (fewer = a hole,
+// since no cell was claimed twice), clears the word and advances the tag
+// for the next call.  The map needs no clearing between calls.
 // Bilinear (spans 1 and 2): a cell map is scattered first (atomicExch into a
 // -1-filled workspace, so double cover and holes are detected), then every
 // output (cell, channel) gathers: span-1 cells are copied, span-2 cells take
@@ -38,36 +45,98 @@ struct Pix4<__nv_bfloat16> {
   }
 };
 
+// Workspace of the merge: a 16-byte header, then one 32-bit word per output
+// cell.  Nearest: header = (tag of the last call, unused, 64-bit CTA count |
+// claimed cells), words = claim map.  Bilinear: the words are the cell map.
+struct MergeHeader {
+  uint32_t last_tag;
+  uint32_t unused;
+  unsigned long long count;   // (CTAs done << 40) | cells claimed
+};
+constexpr int kMergeHeaderBytes = 16;
+
+// Claim tags have bit 31 set (bilinear cell-map entries, -1 aside, have it
+// clear, so a workspace used in both modes never confuses the two) and a
+// 31-bit call counter in 1 .. 2^31 - 2 (never 0, the zeroed map).
+__device__ __forceinline__ uint32_t next_tag(uint32_t last) {
+  const uint32_t g = last & 0x7FFFFFFFu;
+  return 0x80000000u | ((g == 0u || g >= 0x7FFFFFFEu) ? 1u : g + 1u);
+}
+
+// One warp per token, kNearestWarps per CTA (small CTAs spread the latency-
+// bound copy over every SM; 32-warp CTAs measured slower).  A token's area is
+// known once its position and span are read, so the CTA's count goes out
+// first; the claims, the count's atomic and the pixel loads are then in
+// flight together and their results are examined last: the check adds no
+// round trip to the copy's two (position, then pixels).
+constexpr int kNearestWarps = 8;
+
 template <typename T>
-__global__ void __launch_bounds__(kWarpsPerCta * 32)
+__global__ void __launch_bounds__(kNearestWarps * 32)
 merge_nearest_kernel(const T* __restrict__ mixed, int B, int N, const int32_t* __restrict__ pos,
                      const int32_t* __restrict__ span, int fh, int fw, int C, T* __restrict__ out,
-                     unsigned int* status) {
+                     MergeHeader* hdr, uint32_t* __restrict__ claim, unsigned int* status) {
   using PV = typename Pix4<T>::V;
   pdl_wait_then_trigger();
+  __shared__ unsigned int cta_cells;
+  if (threadIdx.x == 0) cta_cells = 0u;
+  const uint32_t last = *reinterpret_cast<volatile uint32_t*>(&hdr->last_tag);
   const int lane = threadIdx.x & 31;
-  const int64_t gwarp = (int64_t)blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
-  if (gwarp >= (int64_t)B * N) return;
-  const int b = (int)(gwarp / N);
-  const int y = pos[gwarp * 2], x = pos[gwarp * 2 + 1], s = span[gwarp];
-  if (s <= 0 || y < 0 || x < 0 || y + s > fh || x + s > fw) {
-    if (lane == 0) raise_status(status, AVITS_ERR_COVERAGE);
-    return;
+  const int64_t gwarp = (int64_t)blockIdx.x * kNearestWarps + (threadIdx.x >> 5);
+  int b = 0, y = 0, x = 0, sp = 0;
+  bool valid = false;
+  if (gwarp < (int64_t)B * N) {
+    b = (int)(gwarp / N);
+    y = pos[gwarp * 2];
+    x = pos[gwarp * 2 + 1];
+    sp = span[gwarp];
+    valid = !(sp <= 0 || y < 0 || x < 0 || y + sp > fh || x + sp > fw);
+    if (!valid && lane == 0) raise_status(status, AVITS_ERR_COVERAGE);
   }
-  const int T4 = C * 4;
-  const T* src = mixed + gwarp * T4;
-  const int tasks = s * s * C;
-  for (int task = lane; task < tasks; task += 32) {
-    const int cell = task / C, c = task - cell * C;
-    const int u = cell / s, v = cell - u * s;
-    const int r0 = (2 * u) / s, r1 = (2 * u + 1) / s;
-    const int c0 = (2 * v) / s, c1 = (2 * v + 1) / s;
-    const T* sc = src + c * 4;
-    const float p00 = load_elem(sc, r0 * 2 + c0), p01 = load_elem(sc, r0 * 2 + c1);
-    const float p10 = load_elem(sc, r1 * 2 + c0), p11 = load_elem(sc, r1 * 2 + c1);
-    const int64_t ocell = (int64_t)b * fh * fw + (int64_t)(y + u) * fw + (x + v);
-    reinterpret_cast<PV*>(out + ocell * T4)[c] = Pix4<T>::make(p00, p01, p10, p11);
+  __syncthreads();   // cta_cells is initialised
+  if (valid && lane == 0) atomicAdd(&cta_cells, (unsigned int)(sp * sp));
+  __syncthreads();
+  unsigned long long v = 0ull;
+  if (threadIdx.x == 0)
+    v = atomicAdd(&hdr->count, (1ull << 40) | (unsigned long long)cta_cells) +
+        ((1ull << 40) | (unsigned long long)cta_cells);
+  const uint32_t tag = next_tag(last);
+  uint32_t old0 = 0u, old1 = 0u;   // claims of this lane (cells lane, lane + 32)
+  bool twice = false;
+  if (valid) {
+    const int64_t base = (int64_t)b * fh * fw;
+    const int area = sp * sp;
+    if (lane < area)
+      old0 = atomicExch(&claim[base + (int64_t)(y + lane / sp) * fw + (x + lane % sp)], tag);
+    if (lane + 32 < area)
+      old1 = atomicExch(&claim[base + (int64_t)(y + (lane + 32) / sp) * fw + (x + (lane + 32) % sp)],
+                        tag);
+    for (int cell = lane + 64; cell < area; cell += 32)   // spans above 8
+      twice |= atomicExch(&claim[base + (int64_t)(y + cell / sp) * fw + (x + cell % sp)], tag) == tag;
+    const int T4 = C * 4;
+    const T* src = mixed + gwarp * T4;
+    const int tasks = area * C;
+    for (int task = lane; task < tasks; task += 32) {
+      const int cell = task / C, c = task - cell * C;
+      const int u = cell / sp, w = cell - u * sp;
+      const int r0 = (2 * u) / sp, r1 = (2 * u + 1) / sp;
+      const int c0 = (2 * w) / sp, c1 = (2 * w + 1) / sp;
+      const T* sc = src + c * 4;
+      const float p00 = load_elem(sc, r0 * 2 + c0), p01 = load_elem(sc, r0 * 2 + c1);
+      const float p10 = load_elem(sc, r1 * 2 + c0), p11 = load_elem(sc, r1 * 2 + c1);
+      const int64_t ocell = base + (int64_t)(y + u) * fw + (x + w);
+      reinterpret_cast<PV*>(out + ocell * T4)[c] = Pix4<T>::make(p00, p01, p10, p11);
+    }
   }
+  if (threadIdx.x == 0 && (v >> 40) == (unsigned long long)gridDim.x) {
+    // every CTA has counted its cells: no cell is claimed twice unless that
+    // is reported, so fewer claimed cells than cells means a hole
+    if ((v & ((1ull << 40) - 1ull)) != (unsigned long long)B * fh * fw)
+      raise_status(status, AVITS_ERR_COVERAGE);
+    hdr->count = 0ull;
+    hdr->last_tag = tag;
+  }
+  if (twice || old0 == tag || old1 == tag) raise_status(status, AVITS_ERR_COVERAGE);
 }
 
 // Cell map entry: the covering token's index, with kSpan2 set when its span
@@ -196,21 +265,23 @@ template <typename T>
 cudaError_t launch_t(const void* mixed, int B, int N, const int32_t* pos, const int32_t* span,
                      int fh, int fw, int C, avits_upmode mode, void* out, void* ws,
                      unsigned int* status, cudaStream_t s) {
+  MergeHeader* hdr = static_cast<MergeHeader*>(ws);
+  uint32_t* words = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + kMergeHeaderBytes);
   if (mode == AVITS_UP_NEAREST) {
     const int64_t warps = (int64_t)B * N;
-    const int grid = (int)((warps + kWarpsPerCta - 1) / kWarpsPerCta);
+    const int grid = (int)((warps + kNearestWarps - 1) / kNearestWarps);
     cudaError_t e = prefer_max_shared<merge_nearest_kernel<T>>();
     if (e != cudaSuccess) return e;
-    e = launch_pdl(merge_nearest_kernel<T>, dim3(grid), dim3(kWarpsPerCta * 32), 0, s,
+    e = launch_pdl(merge_nearest_kernel<T>, dim3(grid), dim3(kNearestWarps * 32), 0, s,
                                static_cast<const T*>(mixed), B, N, pos, span, fh, fw, C,
-                               static_cast<T*>(out), status);
+                               static_cast<T*>(out), hdr, words, status);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
   }
   // three kernels (fill, scatter of the cell map, gather), each a
   // programmatic dependent of the one before: their launches overlap, every
   // kernel waits for its predecessor before touching memory
-  int32_t* map = static_cast<int32_t*>(ws);
+  int32_t* map = reinterpret_cast<int32_t*>(words);
   const int64_t ncell = (int64_t)B * fh * fw;
   cudaError_t e = prefer_max_shared<merge_fill_kernel>();
   if (e == cudaSuccess) e = prefer_max_shared<merge_map_kernel>();
@@ -232,6 +303,10 @@ cudaError_t launch_t(const void* mixed, int B, int N, const int32_t* pos, const 
 }
 
 }  // namespace
+
+size_t merge_workspace_bytes(int B, int fh, int fw) {
+  return kMergeHeaderBytes + sizeof(uint32_t) * (size_t)B * fh * fw;
+}
 
 cudaError_t launch_merge(const void* mixed, avits_dtype dt, int B, int N, const int32_t* pos,
                          const int32_t* span, int fh, int fw, int C, avits_upmode mode,

@@ -65,6 +65,7 @@ avits_status avits_score_spatial_noalloc(const void* q_img, const void* k_all, a
                                          int64_t q_sh, int64_t q_sn, int64_t k_sb, int64_t k_sh,
                                          int64_t k_sn, float softmax_scale, float weight,
                                          int accumulate, float* A, float* lse_opt, void* stream) {
+  AVITS_RANGE();
   t_noalloc_error[0] = '\0';
   if (!q_img || !k_all || !A || dt != AVITS_BF16) return AVITS_ERR_INVALID_ARG;
   if (B <= 0 || H <= 0 || M <= 0 || Nk <= 0 || d <= 0 || L < 0 || L > Nk || Nk < M)
@@ -92,6 +93,17 @@ avits_status avits_score_spatial_noalloc(const void* q_img, const void* k_all, a
   }
   cudaError_t e = scratch_address(&scratch);
   if (e != cudaSuccess) {
+    cudaGetLastError();
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(static_cast<cudaStream_t>(stream), &cap) == cudaSuccess &&
+        cap != cudaStreamCaptureStatusNone)
+      snprintf(t_noalloc_error, sizeof(t_noalloc_error),
+               "avits_score_spatial_noalloc: the first call on a device looks up the scratch "
+               "address and must come before stream capture (%s)", cudaGetErrorString(e));
+    else
+      snprintf(t_noalloc_error, sizeof(t_noalloc_error),
+               "avits_score_spatial_noalloc: scratch address lookup failed (%s)",
+               cudaGetErrorString(e));
     cudaGetLastError();
     return AVITS_ERR_CUDA;
   }

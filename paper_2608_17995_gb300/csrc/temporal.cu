@@ -230,7 +230,15 @@ temporal_staged_kernel(const T* __restrict__ ht, const T* __restrict__ hp, int64
         if (lane == 0) V[t0 + i] = sqrtf(dd) / (sqrtf(pp) + eps);
       }
     }
-    __syncthreads();   // the buffer is reused by the next chunk
+    // the buffer is reused by the next chunk.  After a timeout anywhere in
+    // the CTA no further chunk is issued: thread 0 waits once more (bounded)
+    // for the copies already armed on the barrier, so that none lands in
+    // shared memory after the CTA has exited, and the CTA stops.
+    if (!__syncthreads_and(ok)) {
+      if (threadIdx.x == 0) mbar_wait_bounded(&bar, phase, nullptr, status);
+      __syncthreads();
+      break;
+    }
   }
   if (kOverlapped) asm volatile("griddepcontrol.wait;" ::: "memory");
 }

@@ -68,7 +68,8 @@ class TransitionBuffers:
         self.full = torch.empty(B, self.full_h * self.full_w, tr.C * 4, dtype=dt, **z)
         self.ws = SpatialWorkspace(device)
         mb = avits_merge_final_workspace(self.mode, B, self.full_h, self.full_w)
-        self.merge_ws = torch.empty(max(mb, 4), dtype=torch.uint8, **z) if mb else None
+        # zero-filled before first use (the nearest merge's claim map and counter)
+        self.merge_ws = torch.zeros(max(mb, 16), dtype=torch.uint8, **z) if mb else None
 
     def set_inputs(self, q, k, h_t, h_prev, latent, pos_in=None, span_in=None):
         self.q, self.k, self.h_t, self.h_prev, self.latent = q, k, h_t, h_prev, latent

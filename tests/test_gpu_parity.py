@@ -542,7 +542,7 @@ def _merge(av, mixed, dtype, pos, span, fh, fw, mode, expect_status=0):
     tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
     out = torch.full((B, fh * fw, T), float("nan"), dtype=tdt, device="cuda")
     nb = av.avits_merge_final_workspace(mode, B, fh, fw)
-    ws = torch.empty(max(nb, 1), dtype=torch.uint8, device="cuda") if nb else None
+    ws = torch.zeros(max(nb, 16), dtype=torch.uint8, device="cuda")
     av.avits_merge_final(_dev(mixed, dtype), _dev(pos), _dev(span), fh, fw, out, mode=mode,
                          workspace=ws)
     assert _status(av) == expect_status
@@ -591,19 +591,45 @@ def test_upsample_golden_4x4(av):
         assert out[0, o].tolist() == e["val"]
 
 
-def test_merge_detects_bad_tiling(av, orc):
-    """A token moved onto its neighbour (double cover + hole) raises
-    AVITS_ERR_COVERAGE in bilinear mode; a token outside the frame raises it in
-    nearest mode."""
+@pytest.mark.parametrize("mode", [0, 1])
+def test_merge_detects_bad_tiling(av, orc, mode):
+    """Sec. 3.2 Stage 3 expands tokens that tile the frame exactly once.  In
+    both modes a token moved onto its neighbour (one cell covered twice, one
+    left empty), a duplicated token with the sequence one short of cells (a
+    hole alone: here the last token dropped), and a token outside the frame
+    each raise AVITS_ERR_COVERAGE; a valid tiling right after each bad one
+    still merges cleanly (the workspace state is consistent)."""
     lat = np.random.default_rng(0).standard_normal((1, 16, 8)).astype(np.float32)
     mask = np.zeros((1, 16), np.uint8)
+    mask[0, [5, 10]] = 1
     out, pos, span, _, _ = orc.selective_upsample(lat, 4, 4, mask)
-    bad = pos.copy()
-    bad[0, 1] = bad[0, 0]
-    _merge(av, out, "f32", bad, span, 8, 8, 1, expect_status=6)
-    bad2 = pos.copy()
-    bad2[0, 3] = [7, 7]
-    _merge(av, out, "f32", bad2, span, 8, 8, 0, expect_status=6)
+    import torch
+    B, N, T = out.shape
+    nb = av.avits_merge_final_workspace(mode, B, 8, 8)
+    ws = torch.zeros(nb, dtype=torch.uint8, device="cuda")
+
+    def run(o, p, s, expect):
+        full = torch.full((B, 64, T), float("nan"), dtype=torch.float32, device="cuda")
+        av.avits_merge_final(_dev(o), _dev(p), _dev(s), 8, 8, full, mode=mode, workspace=ws)
+        assert _status(av) == expect
+        return _np(full)
+
+    good, cover = orc.merge_final(out, pos, span, 8, 8,
+                                  mode="nearest" if mode == 0 else "bilinear")
+    assert np.all(cover == 1)
+    moved = pos.copy()
+    moved[0, 1] = moved[0, 0]                       # double cover + hole
+    run(out, moved, span, 6)
+    assert np.array_equal(run(out, pos, span, 0), good)
+    run(out[:, :-1], pos[:, :-1], span[:, :-1], 6)  # hole only
+    assert np.array_equal(run(out, pos, span, 0), good)
+    far = pos.copy()
+    far[0, 3] = [7, 7]                              # outside the frame
+    run(out, far, span, 6)
+    assert np.array_equal(run(out, pos, span, 0), good)
+    dup = np.concatenate([out, out[:, :1]], 1)      # one extra token on cell 0
+    run(dup, np.concatenate([pos, pos[:, :1]], 1), np.concatenate([span, span[:, :1]], 1), 6)
+    assert np.array_equal(run(out, pos, span, 0), good)
 
 
 # ------------------------------------------------------------ end to end ----

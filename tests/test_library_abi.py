@@ -68,9 +68,17 @@ def test_host_validation_rejects_without_launch(lib):
     up[4] = 4
     up[8], up[9], up[13] = P, P, 1
     assert lib.avits_selective_upsample(*up) == UNSUPPORTED
-    # merge: bilinear needs an even frame and a workspace; misaligned output
+    # merge: both modes need a workspace (16-byte aligned, large enough);
+    # bilinear an even frame; misaligned output
     mg = [P, 1, 1, 28, P, P, 8, 8, 1, 2, 1, P, None, 0, None]
     assert lib.avits_merge_final(*mg) == INVALID
+    mg[10] = 0
+    assert lib.avits_merge_final(*mg) == INVALID          # nearest without workspace
+    mg[12], mg[13] = P, 100
+    assert lib.avits_merge_final(*mg) == INVALID          # too small
+    mg[12], mg[13] = ctypes.c_void_p(P.value + 8), 1 << 20
+    assert lib.avits_merge_final(*mg) == INVALID          # misaligned workspace
+    mg[10] = 1
     mg[12], mg[13] = P, 1 << 20
     mg[6] = 7
     assert lib.avits_merge_final(*mg) == INVALID
@@ -80,8 +88,10 @@ def test_host_validation_rejects_without_launch(lib):
 
 
 def test_workspace_queries(lib):
-    assert lib.avits_merge_final_workspace(0, 1, 64, 64) == 0
-    assert lib.avits_merge_final_workspace(1, 2, 64, 64) == 2 * 64 * 64 * 4
+    # a 16-byte header and one 32-bit word per output cell, in both modes
+    assert lib.avits_merge_final_workspace(0, 1, 64, 64) == 16 + 64 * 64 * 4
+    assert lib.avits_merge_final_workspace(1, 2, 64, 64) == 16 + 2 * 64 * 64 * 4
+    assert lib.avits_merge_final_workspace(2, 1, 64, 64) == 0
     assert lib.avits_score_spatial_workspace(0, 1, 2, 256, 288, 64) == 0   # fp32: no workspace
     assert lib.avits_score_spatial_workspace(1, 1, 24, 1024, 1536, 128) > 0
 
@@ -157,3 +167,18 @@ def test_host_validation_of_the_lse_entry(lib):
     assert f(*args(P, 1, 0, 0.125)) == 1
     assert f(*args(P, 1, 32, 0.0)) == 1
     assert f(*args(P, 0, 32, 0.125)) == 2
+
+
+def test_nvtx_ranges_compile(tmp_path):
+    """With AVITS_NVTX the entry points open NVTX ranges (header-only NVTX v3,
+    so nothing to link): the entry-point sources compile with it."""
+    import subprocess
+    from paper_2608_17995_gb300 import _build
+    for src in ("api.cu", "no_alloc.cu"):
+        out = tmp_path / (src + ".o")
+        cmd = [_build.nvcc(), *_build.ARCH, *_build.FLAGS, "-DAVITS_NVTX", "-c",
+               os.path.join(_build.CSRC, src), "-o", str(out)]
+        r = subprocess.run(cmd, stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True)
+        assert r.returncode == 0, r.stdout
+        nm = subprocess.run(["nm", str(out)], stdout=subprocess.PIPE, text=True).stdout
+        assert "nvtx" in nm.lower()

@@ -5,7 +5,9 @@ input/output pointers and a stream and may not allocate there; this entry
 point keeps its scratch in a fixed device array of the library.  These tests
 call it through the C ABI and compare it with avits_score_spatial (which
 takes a caller workspace) on two calls in a row.  The file is named so that
-pytest collects it last.
+pytest collects it last: a run that stops at its first failure has then run
+every other test already.  The tests do not depend on that order (every call
+clears the part of the array it uses), and pass alone in a fresh process.
 """
 import ctypes
 import math
@@ -89,3 +91,44 @@ def test_noalloc_rejects_shapes_beyond_the_array(av):
     lib.avits_score_spatial_noalloc_error.restype = ctypes.c_char_p
     assert b"scratch needed" in lib.avits_score_spatial_noalloc_error()
     assert av.avits_device_status() == 0
+
+
+def test_noalloc_back_to_back_shapes_on_one_stream(av):
+    """Calls with different shapes back to back on one stream (large then
+    small, small then large) each match avits_score_spatial: what the
+    previous call left in the shared array never leaks into the next one."""
+    import torch
+    shapes = [("batched", {}), ("flux1024", dict(G=13, L=77, H=3, k=40)), ("flux1024", {}),
+              ("batched", {})]
+    ins = [_inputs(n, **kw) for n, kw in shapes]
+    refs = []
+    for tr, q, k in ins:
+        ref = torch.full((tr.B, tr.M), float("nan"), device="cuda")
+        av.avits_score_spatial(q, k, tr.L, tr.softmax_scale, ref)
+        refs.append(ref)
+    outs = []
+    st = torch.cuda.Stream()
+    with torch.cuda.stream(st):
+        for tr, q, k in ins:
+            out = torch.full((tr.B, tr.M), float("nan"), device="cuda")
+            av.avits_score_spatial_noalloc(q, k, tr.L, tr.softmax_scale, out, stream=st)
+            outs.append(out)
+    st.synchronize()
+    assert av.avits_device_status() == 0
+    for out, ref in zip(outs, refs):
+        assert not torch.isnan(out).any()
+        np.testing.assert_allclose(out.cpu().numpy(), ref.cpu().numpy(), rtol=RTOL, atol=1e-6)
+
+
+def test_noalloc_limit_covers_the_configurations(av):
+    """On this device (its SM count sets the per-SM scratch) every
+    configuration of the transition fits the fixed array."""
+    from paper_2608_17995_gb300.workloads import make_transition
+    limit = av.avits_score_spatial_noalloc_limit()
+    for name in ("flux1024", "flux2048", "edit", "batched"):
+        tr = make_transition(name)
+        need = av.avits_score_spatial_workspace(av.BF16, tr.B, tr.H, tr.M, tr.Nk, tr.d)
+        assert 0 < need <= limit, (name, need, limit)
+    B, H, M, d, L = 8, 24, 640, 128, 512   # the batched second transition
+    need = av.avits_score_spatial_workspace(av.BF16, B, H, M, L + M, d)
+    assert 0 < need <= limit
