@@ -66,10 +66,28 @@ def _c(a: np.ndarray) -> np.ndarray:
     return a
 
 
+_threads_set = None
+
+
 def threads() -> int:
-    """OpenMP threads the oracle runs on (OMP_NUM_THREADS or all cores)."""
+    """OpenMP threads the oracle runs on (set_threads(), else OMP_NUM_THREADS,
+    else all cores)."""
+    if _threads_set is not None:
+        return _threads_set
     env = os.environ.get("OMP_NUM_THREADS")
     return int(env) if env else (os.cpu_count() or 1)
+
+
+def set_threads(n: int) -> None:
+    """Run the oracle's parallel loops on n threads from now on (the OpenMP
+    runtime's omp_set_num_threads; the arithmetic and its order per token do
+    not depend on it).  Used by the bench to time one thread and all cores."""
+    global _threads_set
+    fn = _load().omp_set_num_threads
+    fn.argtypes = [ctypes.c_int]
+    fn.restype = None
+    fn(int(n))
+    _threads_set = int(n)
 
 
 def score_spatial(q_img: np.ndarray, k_all: np.ndarray, L: int, softmax_scale: float,
