@@ -154,4 +154,52 @@ __device__ __forceinline__ void store_elem(__nv_bfloat16* p, int64_t i, float v)
   p[i] = __float2bfloat16_rn(v);
 }
 
+// The 4 pixels of one channel of a latent token, stored together (the
+// within-token layout is channel, patch row, patch column).
+template <typename T>
+struct Pix4;
+template <>
+struct Pix4<float> {
+  using V = float4;
+  __device__ static V make(float a, float b, float c, float d) { return make_float4(a, b, c, d); }
+};
+template <>
+struct Pix4<__nv_bfloat16> {
+  using V = uint2;
+  __device__ static V make(float a, float b, float c, float d) {
+    const __nv_bfloat162 lo = __floats2bfloat162_rn(a, b);
+    const __nv_bfloat162 hi = __floats2bfloat162_rn(c, d);
+    return make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
+                      *reinterpret_cast<const uint32_t*>(&hi));
+  }
+};
+
+// One 16-byte chunk j of a latent token (channel, patch row, patch column
+// layout) whose channel pixels are taken from a source token's pixels
+// (r0|r1, c0|c1): pixel (0,0) <- (r0,c0), (0,1) <- (r0,c1), (1,0) <- (r1,c0),
+// (1,1) <- (r1,c1).  bf16: a chunk holds two channels; fp32: one.  `src`
+// points at the source token (global or shared memory).
+template <typename T>
+__device__ __forceinline__ uint4 gather_chunk(const void* src, int j, int r0, int r1, int c0,
+                                              int c1);
+template <>
+__device__ __forceinline__ uint4 gather_chunk<__nv_bfloat16>(const void* src, int j, int r0,
+                                                             int r1, int c0, int c1) {
+  const uint16_t* t = static_cast<const uint16_t*>(src);
+  uint32_t w[4];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const uint16_t* ch = t + (2 * j + h) * 4;
+    w[2 * h] = (uint32_t)ch[r0 * 2 + c0] | ((uint32_t)ch[r0 * 2 + c1] << 16);
+    w[2 * h + 1] = (uint32_t)ch[r1 * 2 + c0] | ((uint32_t)ch[r1 * 2 + c1] << 16);
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+template <>
+__device__ __forceinline__ uint4 gather_chunk<float>(const void* src, int j, int r0, int r1,
+                                                     int c0, int c1) {
+  const uint32_t* ch = static_cast<const uint32_t*>(src) + j * 4;
+  return make_uint4(ch[r0 * 2 + c0], ch[r0 * 2 + c1], ch[r1 * 2 + c0], ch[r1 * 2 + c1]);
+}
+
 }  // namespace avits

@@ -25,26 +25,6 @@
 namespace avits {
 namespace {
 
-constexpr int kWarpsPerCta = 8;
-
-template <typename T>
-struct Pix4;
-template <>
-struct Pix4<float> {
-  using V = float4;
-  __device__ static V make(float a, float b, float c, float d) { return make_float4(a, b, c, d); }
-};
-template <>
-struct Pix4<__nv_bfloat16> {
-  using V = uint2;
-  __device__ static V make(float a, float b, float c, float d) {
-    const __nv_bfloat162 lo = __floats2bfloat162_rn(a, b);
-    const __nv_bfloat162 hi = __floats2bfloat162_rn(c, d);
-    return make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
-                      *reinterpret_cast<const uint32_t*>(&hi));
-  }
-};
-
 // Workspace of the merge: a 16-byte header, then one 32-bit word per output
 // cell.  Nearest: header = (tag of the last call, unused, 64-bit CTA count |
 // claimed cells), words = claim map.  Bilinear: the words are the cell map.
@@ -63,33 +43,34 @@ __device__ __forceinline__ uint32_t next_tag(uint32_t last) {
   return 0x80000000u | ((g == 0u || g >= 0x7FFFFFFEu) ? 1u : g + 1u);
 }
 
-// One warp per token, kNearestWarps per CTA (small CTAs spread the latency-
-// bound copy over every SM; 32-warp CTAs measured slower).  A token's area is
-// known once its position and span are read, so the CTA's count goes out
-// first; the claims, the count's atomic and the pixel loads are then in
-// flight together and their results are examined last: the check adds no
-// round trip to the copy's two (position, then pixels).
-constexpr int kNearestWarps = 8;
-
+// Batch-1 sized inputs (at most one token per warp of a capped grid): one
+// warp per token, one pass.  A token's area is known once its position and
+// span are read, so the CTA's count goes out first; the claims, the count's
+// atomic and the pixel loads are then in flight together and their results
+// are examined last: the check adds no round trip to the copy's two
+// (position, then pixels).
 template <typename T>
-__global__ void __launch_bounds__(kNearestWarps * 32)
-merge_nearest_kernel(const T* __restrict__ mixed, int B, int N, const int32_t* __restrict__ pos,
-                     const int32_t* __restrict__ span, int fh, int fw, int C, T* __restrict__ out,
-                     MergeHeader* hdr, uint32_t* __restrict__ claim, unsigned int* status) {
+__global__ void __launch_bounds__(8 * 32)
+merge_nearest_warp_kernel(const T* __restrict__ mixed, int B, int N,
+                          const int32_t* __restrict__ pos, const int32_t* __restrict__ span,
+                          int fh, int fw, int C, T* __restrict__ out, MergeHeader* hdr,
+                          uint32_t* __restrict__ claim, unsigned int* status) {
   using PV = typename Pix4<T>::V;
+  constexpr int kStage = 1024;   // a token of up to 1 KB takes the vector path
   pdl_wait_then_trigger();
+  __shared__ __align__(16) uint8_t stage_all[8 * kStage];
   __shared__ unsigned int cta_cells;
   if (threadIdx.x == 0) cta_cells = 0u;
   const uint32_t last = *reinterpret_cast<volatile uint32_t*>(&hdr->last_tag);
   const int lane = threadIdx.x & 31;
-  const int64_t gwarp = (int64_t)blockIdx.x * kNearestWarps + (threadIdx.x >> 5);
+  const int64_t t = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
   int b = 0, y = 0, x = 0, sp = 0;
   bool valid = false;
-  if (gwarp < (int64_t)B * N) {
-    b = (int)(gwarp / N);
-    y = pos[gwarp * 2];
-    x = pos[gwarp * 2 + 1];
-    sp = span[gwarp];
+  if (t < (int64_t)B * N) {
+    b = (int)(t / N);
+    y = pos[t * 2];
+    x = pos[t * 2 + 1];
+    sp = span[t];
     valid = !(sp <= 0 || y < 0 || x < 0 || y + sp > fh || x + sp > fw);
     if (!valid && lane == 0) raise_status(status, AVITS_ERR_COVERAGE);
   }
@@ -101,11 +82,19 @@ merge_nearest_kernel(const T* __restrict__ mixed, int B, int N, const int32_t* _
     v = atomicAdd(&hdr->count, (1ull << 40) | (unsigned long long)cta_cells) +
         ((1ull << 40) | (unsigned long long)cta_cells);
   const uint32_t tag = next_tag(last);
-  uint32_t old0 = 0u, old1 = 0u;   // claims of this lane (cells lane, lane + 32)
+  uint32_t old0 = 0u, old1 = 0u;   // claims of cells lane and lane + 32
   bool twice = false;
   if (valid) {
     const int64_t base = (int64_t)b * fh * fw;
     const int area = sp * sp;
+    const int T4 = C * 4;
+    const T* src = mixed + t * T4;
+    const int tb = T4 * (int)sizeof(T);
+    const bool vec = (tb & 15) == 0 && tb <= kStage;
+    uint8_t* stage = stage_all + (threadIdx.x >> 5) * kStage;
+    if (vec)
+      for (int q = lane; q < tb / 16; q += 32)
+        reinterpret_cast<uint4*>(stage)[q] = __ldg(reinterpret_cast<const uint4*>(src) + q);
     if (lane < area)
       old0 = atomicExch(&claim[base + (int64_t)(y + lane / sp) * fw + (x + lane % sp)], tag);
     if (lane + 32 < area)
@@ -113,19 +102,31 @@ merge_nearest_kernel(const T* __restrict__ mixed, int B, int N, const int32_t* _
                         tag);
     for (int cell = lane + 64; cell < area; cell += 32)   // spans above 8
       twice |= atomicExch(&claim[base + (int64_t)(y + cell / sp) * fw + (x + cell % sp)], tag) == tag;
-    const int T4 = C * 4;
-    const T* src = mixed + gwarp * T4;
-    const int tasks = area * C;
-    for (int task = lane; task < tasks; task += 32) {
-      const int cell = task / C, c = task - cell * C;
-      const int u = cell / sp, w = cell - u * sp;
-      const int r0 = (2 * u) / sp, r1 = (2 * u + 1) / sp;
-      const int c0 = (2 * w) / sp, c1 = (2 * w + 1) / sp;
-      const T* sc = src + c * 4;
-      const float p00 = load_elem(sc, r0 * 2 + c0), p01 = load_elem(sc, r0 * 2 + c1);
-      const float p10 = load_elem(sc, r1 * 2 + c0), p11 = load_elem(sc, r1 * 2 + c1);
-      const int64_t ocell = base + (int64_t)(y + u) * fw + (x + w);
-      reinterpret_cast<PV*>(out + ocell * T4)[c] = Pix4<T>::make(p00, p01, p10, p11);
+    if (vec) {
+      __syncwarp();
+      const int cpc = tb / 16;
+      for (int q = lane; q < area * cpc; q += 32) {
+        const int cell = q / cpc, j = q - cell * cpc;
+        const int u = cell / sp, w = cell - u * sp;
+        const int r0 = (2 * u) / sp, r1 = (2 * u + 1) / sp;
+        const int c0 = (2 * w) / sp, c1 = (2 * w + 1) / sp;
+        const uint4 chunk = (sp == 1) ? reinterpret_cast<const uint4*>(stage)[j]
+                                      : gather_chunk<T>(stage, j, r0, r1, c0, c1);
+        const int64_t ocell = base + (int64_t)(y + u) * fw + (x + w);
+        reinterpret_cast<uint4*>(out + ocell * T4)[j] = chunk;
+      }
+    } else {
+      for (int task = lane; task < area * C; task += 32) {
+        const int cell = task / C, c = task - cell * C;
+        const int u = cell / sp, w = cell - u * sp;
+        const int r0 = (2 * u) / sp, r1 = (2 * u + 1) / sp;
+        const int c0 = (2 * w) / sp, c1 = (2 * w + 1) / sp;
+        const T* sc = src + c * 4;
+        const float p00 = load_elem(sc, r0 * 2 + c0), p01 = load_elem(sc, r0 * 2 + c1);
+        const float p10 = load_elem(sc, r1 * 2 + c0), p11 = load_elem(sc, r1 * 2 + c1);
+        const int64_t ocell = base + (int64_t)(y + u) * fw + (x + w);
+        reinterpret_cast<PV*>(out + ocell * T4)[c] = Pix4<T>::make(p00, p01, p10, p11);
+      }
     }
   }
   if (threadIdx.x == 0 && (v >> 40) == (unsigned long long)gridDim.x) {
@@ -137,6 +138,140 @@ merge_nearest_kernel(const T* __restrict__ mixed, int B, int N, const int32_t* _
     hdr->last_tag = tag;
   }
   if (twice || old0 == tag || old1 == tag) raise_status(status, AVITS_ERR_COVERAGE);
+}
+
+// Large batches: kLanesPerTok (8) lanes per token (8 x 16 bytes = a
+// 16-channel bf16 token), four tokens in flight per warp; kNearestWarps warps
+// per CTA, at most
+// kNearestCtasPerSm CTAs per SM looping over the tokens (every CTA adds to
+// the one count word, and same-address atomics are serialised: one CTA per
+// 8 tokens of a batch of 64 made the count the bound).  A token's area is
+// known once its position and span are read, so pass 1 sums the CTA's
+// areas and its count goes out before pass 2 copies; the claims, the
+// count's atomic and the pixel loads are then in flight together and their
+// results are examined last.  The first token of each lane group keeps its
+// position in registers between the passes (at batch 1 that is its only
+// token).
+constexpr int kNearestWarps = 8;
+constexpr int kNearestCtasPerSm = 4;
+constexpr int kStageBytes = 512;   // per token slot: a token of up to 512 B takes the vector path
+
+template <typename T, int kLanesPerTok>
+__global__ void __launch_bounds__(kNearestWarps * 32)
+merge_nearest_kernel(const T* __restrict__ mixed, int B, int N, const int32_t* __restrict__ pos,
+                     const int32_t* __restrict__ span, int fh, int fw, int C, T* __restrict__ out,
+                     MergeHeader* hdr, uint32_t* __restrict__ claim, unsigned int* status) {
+  using PV = typename Pix4<T>::V;
+  constexpr int kToksPerWarp = 32 / kLanesPerTok;
+  pdl_wait_then_trigger();
+  __shared__ __align__(16) uint8_t stage_all[kNearestWarps * kToksPerWarp * kStageBytes];
+  __shared__ unsigned int cta_cells;
+  if (threadIdx.x == 0) cta_cells = 0u;
+  const uint32_t last = *reinterpret_cast<volatile uint32_t*>(&hdr->last_tag);
+  const int lane = threadIdx.x & 31, grp = lane / kLanesPerTok, gl = lane % kLanesPerTok;
+  const int warp = threadIdx.x >> 5;
+  const int64_t ntok = (int64_t)B * N;
+  const int64_t tstride = (int64_t)gridDim.x * kNearestWarps * kToksPerWarp;
+  const int64_t t0 = ((int64_t)blockIdx.x * kNearestWarps + warp) * kToksPerWarp + grp;
+  // pass 1: validate the tokens and sum their areas
+  unsigned int cells = 0u;
+  int y0 = 0, x0 = 0, s0 = 0;
+  for (int64_t t = t0; t < ntok; t += tstride) {
+    const int y = pos[t * 2], x = pos[t * 2 + 1], sp = span[t];
+    if (t == t0) { y0 = y; x0 = x; s0 = sp; }
+    if (sp <= 0 || y < 0 || x < 0 || y + sp > fh || x + sp > fw) {
+      if (gl == 0) raise_status(status, AVITS_ERR_COVERAGE);
+    } else if (gl == 0) {
+      cells += (unsigned int)(sp * sp);
+    }
+  }
+  __syncthreads();   // cta_cells is initialised
+  if (cells) atomicAdd(&cta_cells, cells);
+  __syncthreads();
+  unsigned long long v = 0ull;
+  if (threadIdx.x == 0)
+    v = atomicAdd(&hdr->count, (1ull << 40) | (unsigned long long)cta_cells) +
+        ((1ull << 40) | (unsigned long long)cta_cells);
+  const uint32_t tag = next_tag(last);
+  bool twice = false;
+  uint8_t* stage = stage_all + (warp * kToksPerWarp + grp) * kStageBytes;
+  const int T4 = C * 4;
+  const int tb = T4 * (int)sizeof(T);
+  const bool vec = (tb & 15) == 0 && tb <= kStageBytes;
+  // pass 2: claim the cells and copy (all lanes of the warp run the same
+  // number of iterations, so the warp-wide syncs below are safe)
+  const int64_t iters = (ntok - (t0 - grp) + tstride - 1) / tstride;
+  for (int64_t it = 0; it < iters; ++it) {
+    const int64_t t = t0 + it * tstride;
+    const bool have = t < ntok;
+    int y = 0, x = 0, sp = 0;
+    if (have) {
+      if (it == 0) { y = y0; x = x0; sp = s0; }
+      else { y = pos[t * 2]; x = pos[t * 2 + 1]; sp = span[t]; }
+    }
+    const bool ok = have && !(sp <= 0 || y < 0 || x < 0 || y + sp > fh || x + sp > fw);
+    const T* src = mixed + (have ? t : 0) * T4;
+    if (vec) {
+      __syncwarp();   // the slot's previous token is read
+      if (ok)
+        for (int q = gl; q < tb / 16; q += kLanesPerTok)
+          reinterpret_cast<uint4*>(stage)[q] = __ldg(reinterpret_cast<const uint4*>(src) + q);
+      __syncwarp();
+    }
+    if (!ok) continue;
+    const int b = (int)(t / N);
+    const int64_t base = (int64_t)b * fh * fw;
+    const int area = sp * sp;
+    // claims of cells gl and gl + kLanesPerTok are examined after the copy,
+    // so their round trip overlaps it
+    uint32_t old0 = 0u, old1 = 0u;
+    if (gl < area)
+      old0 = atomicExch(&claim[base + (int64_t)(y + gl / sp) * fw + (x + gl % sp)], tag);
+    if (gl + kLanesPerTok < area) {
+      const int c1 = gl + kLanesPerTok;
+      old1 = atomicExch(&claim[base + (int64_t)(y + c1 / sp) * fw + (x + c1 % sp)], tag);
+    }
+    for (int cell = gl + 2 * kLanesPerTok; cell < area; cell += kLanesPerTok)
+      twice |= atomicExch(&claim[base + (int64_t)(y + cell / sp) * fw + (x + cell % sp)], tag) == tag;
+    if (vec) {
+      // 16-byte output chunks: cell (u, w) of the token's s x s block takes,
+      // for channel c, the token's pixels (r0|r1, c0|c1); chunks of one cell
+      // are consecutive, so the stores are coalesced
+      const int cpc = tb / 16;
+      for (int q = gl; q < area * cpc; q += kLanesPerTok) {
+        const int cell = q / cpc, j = q - cell * cpc;
+        const int u = cell / sp, w = cell - u * sp;
+        const int r0 = (2 * u) / sp, r1 = (2 * u + 1) / sp;
+        const int c0 = (2 * w) / sp, c1 = (2 * w + 1) / sp;
+        const uint4 chunk = (sp == 1) ? reinterpret_cast<const uint4*>(stage)[j]
+                                      : gather_chunk<T>(stage, j, r0, r1, c0, c1);
+        const int64_t ocell = base + (int64_t)(y + u) * fw + (x + w);
+        reinterpret_cast<uint4*>(out + ocell * T4)[j] = chunk;
+      }
+    } else {
+      for (int task = gl; task < area * C; task += kLanesPerTok) {
+        const int cell = task / C, c = task - cell * C;
+        const int u = cell / sp, w = cell - u * sp;
+        const int r0 = (2 * u) / sp, r1 = (2 * u + 1) / sp;
+        const int c0 = (2 * w) / sp, c1 = (2 * w + 1) / sp;
+        const T* sc = src + c * 4;
+        const float p00 = load_elem(sc, r0 * 2 + c0), p01 = load_elem(sc, r0 * 2 + c1);
+        const float p10 = load_elem(sc, r1 * 2 + c0), p11 = load_elem(sc, r1 * 2 + c1);
+        const int64_t ocell = base + (int64_t)(y + u) * fw + (x + w);
+        reinterpret_cast<PV*>(out + ocell * T4)[c] = Pix4<T>::make(p00, p01, p10, p11);
+      }
+    }
+    twice |= old0 == tag || old1 == tag;
+  }
+  if (threadIdx.x == 0 && (v >> 40) == (unsigned long long)gridDim.x) {
+    // every CTA has counted its cells: no cell is claimed twice unless that
+    // is reported, so fewer claimed cells than cells means a hole
+    if ((v & ((1ull << 40) - 1ull)) != (unsigned long long)B * fh * fw)
+      raise_status(status, AVITS_ERR_COVERAGE);
+    hdr->count = 0ull;
+    hdr->last_tag = tag;
+  }
+  if (twice) raise_status(status, AVITS_ERR_COVERAGE);   // a cell claimed twice
 }
 
 // Cell map entry: the covering token's index, with kSpan2 set when its span
@@ -268,11 +403,26 @@ cudaError_t launch_t(const void* mixed, int B, int N, const int32_t* pos, const 
   MergeHeader* hdr = static_cast<MergeHeader*>(ws);
   uint32_t* words = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + kMergeHeaderBytes);
   if (mode == AVITS_UP_NEAREST) {
-    const int64_t warps = (int64_t)B * N;
-    const int grid = (int)((warps + kNearestWarps - 1) / kNearestWarps);
-    cudaError_t e = prefer_max_shared<merge_nearest_kernel<T>>();
+    const int64_t ntok = (int64_t)B * N;
+    int dev = 0, sms = 0;
+    cudaError_t e0 = cudaGetDevice(&dev);
+    if (e0 == cudaSuccess) e0 = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e0 != cudaSuccess) return e0;
+    const int64_t cap = (int64_t)std::max(1, sms) * kNearestCtasPerSm;
+    cudaError_t e = prefer_max_shared<merge_nearest_warp_kernel<T>>();
+    if (e == cudaSuccess) e = prefer_max_shared<merge_nearest_kernel<T, 8>>();
     if (e != cudaSuccess) return e;
-    e = launch_pdl(merge_nearest_kernel<T>, dim3(grid), dim3(kNearestWarps * 32), 0, s,
+    if (ntok <= cap * kNearestWarps) {
+      // one warp per token, one pass (latency-bound sizes)
+      e = launch_pdl(merge_nearest_warp_kernel<T>, dim3((unsigned)((ntok + 7) / 8)),
+                     dim3(8 * 32), 0, s, static_cast<const T*>(mixed), B, N, pos, span, fh, fw,
+                     C, static_cast<T*>(out), hdr, words, status);
+      if (e != cudaSuccess) return e;
+      return cudaGetLastError();
+    }
+    const int64_t per_cta = (int64_t)kNearestWarps * 4;
+    const int grid = (int)std::min<int64_t>((ntok + per_cta - 1) / per_cta, cap);
+    e = launch_pdl(merge_nearest_kernel<T, 8>, dim3(grid), dim3(kNearestWarps * 32), 0, s,
                                static_cast<const T*>(mixed), B, N, pos, span, fh, fw, C,
                                static_cast<T*>(out), hdr, words, status);
     if (e != cudaSuccess) return e;

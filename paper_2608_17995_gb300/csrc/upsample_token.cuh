@@ -9,32 +9,15 @@
 //                broadcasts the pixel; bilinear applies the fixed 0.25 / 0.75
 //                weights of a half-pixel-centred 2x resize with edge clamping,
 //                reading neighbouring pixels from the dense input latent.
-// Lanes split the (child, channel) work; each writes the 4 pixels of one
-// channel of one child, and lanes 0-3 write the position / span / source maps.
+// Nearest with 16-byte token rows: each lane writes whole 16-byte chunks
+// (coalesced); otherwise lanes split the (child, channel) work, each writing
+// the 4 pixels of one channel of one child.  Lanes 0-3 write the position /
+// span / source maps.
 #pragma once
 
 #include "avits_common.cuh"
 
 namespace avits {
-
-template <typename T>
-struct Pix4;   // 4 pixels of one channel, stored together
-
-template <>
-struct Pix4<float> {
-  using V = float4;
-  __device__ static V make(float a, float b, float c, float d) { return make_float4(a, b, c, d); }
-};
-template <>
-struct Pix4<__nv_bfloat16> {
-  using V = uint2;
-  __device__ static V make(float a, float b, float c, float d) {
-    const __nv_bfloat162 lo = __floats2bfloat162_rn(a, b);
-    const __nv_bfloat162 hi = __floats2bfloat162_rn(c, d);
-    return make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
-                      *reinterpret_cast<const uint32_t*>(&hi));
-  }
-};
 
 __device__ __forceinline__ void bil_axis(int P, int n, int& r0, int& r1, float& w0, float& w1) {
   const int m = P >> 1;
@@ -105,10 +88,56 @@ __device__ __forceinline__ void upsample_token(const UpsampleArgs<T>& u, const S
   }
   const T* src = rows.row(b, i);
   const int64_t out_tok0 = (int64_t)b * u.n_out + o;
-  if (!sel) {
+  const int tb = T4 * (int)sizeof(T);
+  if (!kBilinear && (tb & 15) == 0) {
+    // 16-byte chunks: a deferred token is copied, a selected one gives each
+    // child (a, b) the chunk whose channel pixels all equal the parent's
+    // pixel (a, b); one chunk per lane (bf16, 16 channels: 32 lanes, 4 children)
+    const int cpc = tb / 16;
+    if (!sel) {
+      uint4* dst = reinterpret_cast<uint4*>(u.out + out_tok0 * T4);
+      for (int q = lane; q < cpc; q += 32) dst[q] = reinterpret_cast<const uint4*>(src)[q];
+    } else {
+      for (int q = lane; q < 4 * cpc; q += 32) {
+        const int child = q / cpc, j = q - child * cpc;
+        const int a = child >> 1, bb = child & 1;
+        reinterpret_cast<uint4*>(u.out + (out_tok0 + child) * T4)[j] =
+            gather_chunk<T>(src, j, a, a, bb, bb);
+      }
+    }
+  } else if (!sel) {
     PV* dst = reinterpret_cast<PV*>(u.out + out_tok0 * T4);
     const PV* sp = reinterpret_cast<const PV*>(src);
     for (int c = lane; c < C; c += 32) dst[c] = sp[c];
+  } else {
+    for (int task = lane; task < 4 * C; task += 32) {
+      const int child = task / C, c = task - child * C;
+      const int a = child >> 1, bb = child & 1;
+      PV v;
+      if (!kBilinear) {
+        const float p = load_elem(src, c * 4 + a * 2 + bb);
+        v = Pix4<T>::make(p, p, p, p);
+      } else {
+        const int IH = 2 * gh, IW = 2 * gw;
+        float r[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int ph = q >> 1, pw = q & 1;
+          int r0, r1, c0, c1;
+          float wy0, wy1, wx0, wx1;
+          bil_axis(4 * y + 2 * a + ph, IH, r0, r1, wy0, wy1);
+          bil_axis(4 * x + 2 * bb + pw, IW, c0, c1, wx0, wx1);
+          auto pix = [&](int R, int Q) {
+            return load_elem(rows.row(b, (R >> 1) * gw + (Q >> 1)), c * 4 + (R & 1) * 2 + (Q & 1));
+          };
+          r[q] = bil_combine(pix(r0, c0), pix(r0, c1), pix(r1, c0), pix(r1, c1), wy0, wy1, wx0, wx1);
+        }
+        v = Pix4<T>::make(r[0], r[1], r[2], r[3]);
+      }
+      reinterpret_cast<PV*>(u.out + (out_tok0 + child) * T4)[c] = v;
+    }
+  }
+  if (!sel) {
     if (lane == 0) {
       u.out_pos[out_tok0 * 2] = 2 * y;
       u.out_pos[out_tok0 * 2 + 1] = 2 * x;
@@ -117,32 +146,6 @@ __device__ __forceinline__ void upsample_token(const UpsampleArgs<T>& u, const S
       u.out_src_sub[out_tok0] = -1;
     }
     return;
-  }
-  for (int task = lane; task < 4 * C; task += 32) {
-    const int child = task / C, c = task - child * C;
-    const int a = child >> 1, bb = child & 1;
-    PV v;
-    if (!kBilinear) {
-      const float p = load_elem(src, c * 4 + a * 2 + bb);
-      v = Pix4<T>::make(p, p, p, p);
-    } else {
-      const int IH = 2 * gh, IW = 2 * gw;
-      float r[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int ph = q >> 1, pw = q & 1;
-        int r0, r1, c0, c1;
-        float wy0, wy1, wx0, wx1;
-        bil_axis(4 * y + 2 * a + ph, IH, r0, r1, wy0, wy1);
-        bil_axis(4 * x + 2 * bb + pw, IW, c0, c1, wx0, wx1);
-        auto pix = [&](int R, int Q) {
-          return load_elem(rows.row(b, (R >> 1) * gw + (Q >> 1)), c * 4 + (R & 1) * 2 + (Q & 1));
-        };
-        r[q] = bil_combine(pix(r0, c0), pix(r0, c1), pix(r1, c0), pix(r1, c1), wy0, wy1, wx0, wx1);
-      }
-      v = Pix4<T>::make(r[0], r[1], r[2], r[3]);
-    }
-    reinterpret_cast<PV*>(u.out + (out_tok0 + child) * T4)[c] = v;
   }
   if (lane < 4) {
     const int a = lane >> 1, bb = lane & 1;
