@@ -338,7 +338,7 @@ def test_spatiotemporal_matches_separate_calls(av, orc, name):
 
 # ------------------------------------------------------------ temporal ----
 
-@pytest.mark.parametrize("name", ["tiny", "flux1024", "edit"])
+@pytest.mark.parametrize("name", ["tiny", "flux1024", "edit", "flux2048", "batched"])
 def test_temporal_configs(av, orc, name):
     import torch
     from paper_2608_17995_gb300.workloads import make_transition
@@ -634,19 +634,29 @@ def test_merge_detects_bad_tiling(av, orc, mode):
 
 # ------------------------------------------------------------ end to end ----
 
-@pytest.mark.parametrize("name", ["tiny", "flux1024"])
-def test_transition_end_to_end(av, orc, name):
-    """The whole path on the device; selected sets may differ from the oracle's
-    only at tokens whose oracle score is within 1e-3 of the k-th score."""
-    import torch
+@pytest.mark.parametrize("name,mode", [("tiny", "nearest"), ("flux1024", "nearest"),
+                                       ("flux1024", "bilinear"), ("flux2048", "nearest"),
+                                       ("edit", "nearest"), ("batched", "nearest")])
+def test_transition_end_to_end(av, orc, name, mode):
+    """The whole path on the device (both scores in one call, selection +
+    upsample in one launch, merge) against the oracle's transition computed
+    from the same inputs on every image row: A and V within the score
+    tolerance; selected sets may differ from the oracle's only at tokens whose
+    oracle score is within 1e-3 of the k-th score; the upsample and merge
+    are bit-exact given the device's own selection.  Every configuration,
+    including the editing shape (alpha = 0.6, k = 205, 4096 reference keys in
+    the softmax) and the batched schedule's first transition (B = 8)."""
     from paper_2608_17995_gb300.pipeline import TransitionBuffers
     from paper_2608_17995_gb300.workloads import make_transition
     tr = make_transition(name)
-    buf = TransitionBuffers(tr)
+    buf = TransitionBuffers(tr, mode=mode)
     buf.run()
     assert _status(av) == 0
     A_o, _, _ = orc.score_spatial(tr.q_img, tr.k_all, tr.L, tr.softmax_scale)
     V_o = orc.score_temporal(tr.h_t, tr.h_prev)
+    rtol = F32_TOL if tr.dtype == "f32" else BF16_RTOL
+    np.testing.assert_allclose(_np(buf.A), A_o, rtol=rtol, atol=1e-6)
+    np.testing.assert_allclose(_np(buf.V), V_o, rtol=rtol, atol=1e-7)
     S_o = orc.fuse(A_o, V_o, tr.alpha)
     sel_o, _, _ = orc.topk(S_o, tr.k)
     sel_g = _np(buf.sel_idx)[:, :tr.k]
@@ -654,13 +664,41 @@ def test_transition_end_to_end(av, orc, name):
         kth = np.sort(S_o[b])[::-1][tr.k - 1]
         diff = set(sel_g[b].tolist()) ^ set(sel_o[b].tolist())
         for i in diff:
-            assert abs(float(S_o[b, i]) - float(kth)) < 1e-3, (i, S_o[b, i], kth)
+            assert abs(float(S_o[b, i]) - float(kth)) < 1e-3, (b, i, S_o[b, i], kth)
     # the rest of the path is exact given the device's own selection
-    o = orc.selective_upsample(tr.latent, tr.grid_h, tr.grid_w, _np(buf.sel_mask))
+    o = orc.selective_upsample(tr.latent, tr.grid_h, tr.grid_w, _np(buf.sel_mask), mode=mode)
     assert np.array_equal(_bits(_np(buf.mixed)), _bits(o[0]))
     assert np.array_equal(_np(buf.pos), o[1]) and np.array_equal(_np(buf.span), o[2])
-    full_o, _ = orc.merge_final(o[0], o[1], o[2], 2 * tr.grid_h, 2 * tr.grid_w)
+    full_o, cover = orc.merge_final(o[0], o[1], o[2], 2 * tr.grid_h, 2 * tr.grid_w, mode=mode)
+    assert np.all(cover == 1)
     assert np.array_equal(_bits(_np(buf.full)), _bits(full_o))
+
+
+@pytest.mark.parametrize("name,mode", [("flux2048", "nearest"), ("edit", "nearest"),
+                                       ("g40", "bilinear"), ("g40", "nearest")])
+def test_select_upsample_fused_vs_oracle(av, orc, name, mode):
+    """avits_select_upsample (one launch) against the oracle given the same
+    scores A, V: the fused score S, sel_idx, mask and tok_offset, the mixed
+    sequence and its maps all bit-exact (M = 4096 at FLUX-2048, 1600 at
+    G = 40; the editing shape's alpha = 0.6 and k = 205)."""
+    from paper_2608_17995_gb300.pipeline import TransitionBuffers
+    from paper_2608_17995_gb300.workloads import make_transition
+    tr = make_transition("flux1024", G=40, k=480) if name == "g40" else make_transition(name)
+    buf = TransitionBuffers(tr, mode=mode)
+    buf.spatial()
+    buf.temporal()
+    buf.select_upsample()
+    assert _status(av) == 0
+    A, V = _np(buf.A), _np(buf.V)
+    S_o = orc.fuse(A, V, tr.alpha)
+    assert np.array_equal(_bits(_np(buf.S)), _bits(S_o))
+    sel_o, mask_o, off_o = orc.topk(S_o, tr.k)
+    assert np.array_equal(_np(buf.sel_idx)[:, :tr.k], sel_o)
+    assert np.array_equal(_np(buf.sel_mask), mask_o) and np.array_equal(_np(buf.tok_offset), off_o)
+    o = orc.selective_upsample(tr.latent, tr.grid_h, tr.grid_w, mask_o, mode=mode)
+    assert np.array_equal(_bits(_np(buf.mixed)), _bits(o[0]))
+    assert np.array_equal(_np(buf.pos), o[1]) and np.array_equal(_np(buf.span), o[2])
+    assert np.array_equal(_np(buf.src_tok), o[3]) and np.array_equal(_np(buf.src_sub), o[4])
 
 
 def _fused_vs_separate(av, buf, perturb=None, k=None):
