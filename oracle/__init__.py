@@ -136,6 +136,38 @@ def score_spatial(q_img: np.ndarray, k_all: np.ndarray, L: int, softmax_scale: f
     return A, mass, lse
 
 
+def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, L: int, softmax_scale: float,
+              weight: float = 1.0, A_in: Optional[np.ndarray] = None,
+              rows: Optional[Sequence[int]] = None):
+    """Eq. 4-5: the joint-attention forward O = softmax(scale Q K^T) V of a
+    double-stream block, q [B,H,Mq,d], k and v [B,H,Nk,d] (contiguous), the
+    text keys first.  Returns (O [B,H,Mq,d] fp64, lse [B,H,Mq,2] fp64 (all
+    keys, text keys), mass [B,H,Mq] fp64 (Eq. 5), A [B,Mq] fp32 (Eq. 3)).
+    With ``rows`` only those flat b*Mq+i rows are computed (others are 0)."""
+    lib = _load()
+    dt = _dtype_code(q)
+    if _dtype_code(k) != dt or _dtype_code(v) != dt:
+        raise TypeError("q, k and v dtypes differ")
+    B, H, Mq, d = q.shape
+    Nk = k.shape[2]
+    if k.shape != (B, H, Nk, d) or v.shape != (B, H, Nk, d):
+        raise ValueError("k and v must be [B,H,Nk,d] with the q's B, H and d")
+    q, k, v = _c(q), _c(k), _c(v)
+    O = np.zeros((B, H, Mq, d), np.float64)
+    lse = np.zeros((B, H, Mq, 2), np.float64)
+    mass = np.zeros((B, H, Mq), np.float64)
+    A = np.zeros((B, Mq), np.float32) if A_in is None else np.array(A_in, np.float32, copy=True)
+    rows_arr = None if rows is None else np.ascontiguousarray(np.asarray(rows, np.int32))
+    fn = lib.avits_oracle_attention
+    fn.restype = ctypes.c_int
+    rc = fn(_p(q), _p(k), _p(v), dt, B, H, Mq, Nk, L, d, ctypes.c_double(softmax_scale),
+            ctypes.c_double(weight), 0 if A_in is None else 1, _p(rows_arr),
+            0 if rows_arr is None else len(rows_arr), _p(O), _p(lse), _p(mass), _p(A))
+    if rc != 0:
+        raise ValueError("oracle attention: bad arguments (%d)" % rc)
+    return O, lse, mass, A
+
+
 def score_temporal(h_t: np.ndarray, h_prev: np.ndarray, eps: float = 1e-6) -> np.ndarray:
     lib = _load()
     dt = _dtype_code(h_t)

@@ -10,6 +10,8 @@
  *   spatial   Sec. 3.3.1, Eq. 3 (head mean of text attention mass) with the
  *             joint-attention extraction of Eq. 4-5 (softmax of Q K^T/sqrt(d)
  *             over the concatenated [text; image] keys, image rows, text cols)
+ *   attention Eq. 4-5, the block's joint attention O = softmax(Q K^T/sqrt(d)) V
+ *             with the logsumexp over all and over the text keys and Eq. 3
  *   temporal  Sec. 3.3.2 — the relative two-snapshot change used by this
  *             build, and Eq. 6-7 (unbiased step variance, channel mean)
  *   fuse      Sec. 3.3.3, min-max normalisation and Eq. 8
@@ -24,7 +26,8 @@
  * which is fp32 as the library's outputs are.  Build with -ffp-contract=off.
  *
  * Parity pins (tests/test_oracle_pins.py): brute-force NumPy softmax and a
- * full sort on small inputs, closed forms (Q = 0, one hot logit, h_t = c h_prev,
+ * full sort on small inputs, torch's CPU scaled_dot_product_attention in
+ * fp64, closed forms (Q = 0, one hot logit, h_t = c h_prev,
  * two-snapshot variance), invariants (mass in [0,1], |S| = k, N_out = M + 3k,
  * exact tiling), the hand-worked 4x4 example in tests/golden/, and torch's
  * bilinear / nearest resize on dense grids.
@@ -140,6 +143,81 @@ int avits_oracle_score_spatial(const void* q, const void* k, int dtype, int B, i
     if (A) A[flat] = accumulate ? (float)((double)A[flat] + a) : (float)a;
     free(P);
     free(qv);
+  }
+  return bad ? OR_BAD_ARG : OR_OK;
+}
+
+/* ---------------------------------------------------------------------------
+ * Joint-attention forward of a double-stream block, Eq. 4-5 (Sec. 3.3.1):
+ * the block's own attention over the concatenated [text; image] sequence,
+ *   O_i = sum_j softmax_j(scale * q_i . k_j) v_j,
+ * with, from the same softmax row, the logsumexp over all keys, the
+ * logsumexp over the text keys (the first L) and the text mass that Eq. 5
+ * extracts; A_i is the mean of that mass over the heads (Eq. 3), times
+ * `weight`, added to A_i when `accumulate`.  Query rows are whatever the
+ * caller passes (text and image rows of the joint sequence alike); A is
+ * given for every row.
+ *
+ * q [B,H,Mq,d], k and v [B,H,Nk,d], all contiguous.
+ * rows: NULL for all B*Mq rows, else `nrows` flat indices b*Mq + i.
+ * o_out [B,H,Mq,d] fp64, lse_out [B,H,Mq,2] fp64 (all, text; -inf when the
+ * row has no text key), mass_out [B,H,Mq] fp64, A [B,Mq] fp32; each may be
+ * NULL.
+ * ------------------------------------------------------------------------- */
+int avits_oracle_attention(const void* q, const void* k, const void* v, int dtype, int B, int H,
+                           int Mq, int Nk, int L, int d, double scale, double weight,
+                           int accumulate, const int32_t* rows, int nrows, double* o_out,
+                           double* lse_out, double* mass_out, float* A) {
+  if (B <= 0 || H <= 0 || Mq <= 0 || Nk <= 0 || d <= 0 || L < 0 || L > Nk) return OR_BAD_ARG;
+  int n = rows ? nrows : B * Mq;
+  int bad = 0;
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int r = 0; r < n; ++r) {
+    int flat = rows ? rows[r] : r;
+    if (flat < 0 || flat >= B * Mq) { bad = 1; continue; }
+    int b = flat / Mq, i = flat % Mq;
+    double* w = (double*)malloc(sizeof(double) * (size_t)Nk);
+    double* ov = (double*)malloc(sizeof(double) * (size_t)d);
+    double head_sum = 0.0;
+    for (int h = 0; h < H; ++h) {
+      const int64_t qoff = (((int64_t)b * H + h) * Mq + i) * d;
+      const int64_t kv0 = ((int64_t)b * H + h) * (int64_t)Nk * d;
+      /* logits P = scale * Q K^T (the row of query i) */
+      for (int j = 0; j < Nk; ++j) {
+        double dot = 0.0;
+        for (int c = 0; c < d; ++c)
+          dot += get_elem(q, dtype, qoff + c) * get_elem(k, dtype, kv0 + (int64_t)j * d + c);
+        w[j] = scale * dot;
+      }
+      /* softmax over all keys (the row maximum subtracted first) */
+      double mx = -INFINITY;
+      for (int j = 0; j < Nk; ++j) if (w[j] > mx) mx = w[j];
+      double z = 0.0, ztxt = 0.0;
+      for (int j = 0; j < Nk; ++j) {
+        w[j] = exp(w[j] - mx);
+        z += w[j];
+        if (j < L) ztxt += w[j];
+      }
+      /* O = softmax(P) V */
+      for (int c = 0; c < d; ++c) ov[c] = 0.0;
+      for (int j = 0; j < Nk; ++j) {
+        const double a = w[j] / z;
+        for (int c = 0; c < d; ++c) ov[c] += a * get_elem(v, dtype, kv0 + (int64_t)j * d + c);
+      }
+      const double mass = ztxt / z;   /* Eq. 5: this row's text columns of the softmax */
+      head_sum += mass;
+      const int64_t row = ((int64_t)b * H + h) * Mq + i;
+      if (o_out) for (int c = 0; c < d; ++c) o_out[row * d + c] = ov[c];
+      if (lse_out) {
+        lse_out[row * 2 + 0] = mx + log(z);
+        lse_out[row * 2 + 1] = ztxt > 0 ? mx + log(ztxt) : -INFINITY;
+      }
+      if (mass_out) mass_out[row] = mass;
+    }
+    double a = weight * (head_sum / (double)H);   /* Eq. 3: mean over heads */
+    if (A) A[flat] = accumulate ? (float)((double)A[flat] + a) : (float)a;
+    free(w);
+    free(ov);
   }
   return bad ? OR_BAD_ARG : OR_OK;
 }

@@ -171,6 +171,110 @@ def test_spatial_text_mask(oracle_mod, seed, B, H, M, Nk, d):
     np.testing.assert_allclose(mass_p, mass, rtol=0, atol=1e-12)
 
 
+# ------------------------------------------------ joint-attention forward (Eq. 4-5)
+
+@pytest.mark.parametrize("seed,B,H,Mq,Nk,L,d,dt", [
+    (0, 1, 2, 9, 13, 4, 8, "f32"),
+    (1, 2, 3, 17, 40, 12, 16, "bf16"),
+    (2, 1, 1, 5, 7, 0, 4, "f32"),       # no text key
+    (3, 1, 2, 6, 6, 6, 8, "f32"),       # every key a text key
+])
+def test_attention_matches_torch_sdpa(oracle_mod, seed, B, H, Mq, Nk, L, d, dt):
+    """The forward's O against torch's CPU scaled_dot_product_attention in fp64
+    (an independent library routine), its logsumexp against torch.logsumexp of
+    the logits, and mass / lse_txt / A against the spatial-score function,
+    which is pinned on its own above (Eq. 3, 5)."""
+    import torch
+    rng = np.random.default_rng(seed)
+    q = rng.standard_normal((B, H, Mq, d)).astype(np.float32)
+    k = rng.standard_normal((B, H, Nk, d)).astype(np.float32)
+    v = rng.standard_normal((B, H, Nk, d)).astype(np.float32)
+    if dt == "bf16":
+        from paper_2608_17995_gb300.workloads import to_bf16_bits
+        q, k, v = to_bf16_bits(q), to_bf16_bits(k), to_bf16_bits(v)
+    scale = 1.0 / math.sqrt(d)
+    O, lse, mass, A = oracle_mod.attention(q, k, v, L, scale)
+    tq, tk, tv = (torch.tensor(as_f32(x), dtype=torch.float64) for x in (q, k, v))
+    ref = torch.nn.functional.scaled_dot_product_attention(tq, tk, tv, scale=scale).numpy()
+    np.testing.assert_allclose(O, ref, rtol=1e-12, atol=1e-12)
+    logits = torch.einsum("bhid,bhjd->bhij", tq, tk) * scale
+    np.testing.assert_allclose(lse[..., 0], torch.logsumexp(logits, -1).numpy(), rtol=1e-12,
+                               atol=1e-12)
+    A_s, mass_s, lse_s = oracle_mod.score_spatial(q, k, L, scale)
+    np.testing.assert_allclose(mass, mass_s, rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(lse[..., 1], lse_s[..., 1], rtol=1e-12, atol=1e-12)
+    np.testing.assert_array_equal(A, A_s)
+    if L == 0:
+        assert np.all(np.isneginf(lse[..., 1])) and np.all(mass == 0)
+    if L == Nk:
+        np.testing.assert_allclose(mass, 1.0, rtol=0, atol=1e-15)
+
+
+def test_attention_closed_forms(oracle_mod):
+    """Closed forms that catch a missing normalisation, swapped k / v, a wrong
+    scale and a transposed product:
+      v_j = c for every key -> O_i = c (the softmax weights sum to one);
+      Q = 0 -> uniform weights, O_i = mean_j v_j, lse = log Nk, mass = L/Nk;
+      one logit a on key 0 (others 0) ->
+        O_i = (e^a v_0 + sum_{j>0} v_j) / (e^a + Nk - 1)."""
+    rng = np.random.default_rng(11)
+    B, H, Mq, Nk, L, d = 1, 2, 4, 6, 2, 4
+    q = rng.standard_normal((B, H, Mq, d)).astype(np.float32)
+    k = rng.standard_normal((B, H, Nk, d)).astype(np.float32)
+    c = np.array([0.5, -2.0, 3.25, 1.0], np.float32)
+    v = np.broadcast_to(c, (B, H, Nk, d)).astype(np.float32).copy()
+    O, _, _, _ = oracle_mod.attention(q, k, v, L, 0.7)
+    np.testing.assert_allclose(O, np.broadcast_to(c, O.shape), rtol=1e-14, atol=1e-14)
+
+    v = rng.standard_normal((B, H, Nk, d)).astype(np.float32)
+    O, lse, mass, A = oracle_mod.attention(np.zeros_like(q), k, v, L, 0.7)
+    np.testing.assert_allclose(O, np.broadcast_to(v.astype(np.float64).mean(2, keepdims=True),
+                                                  O.shape), rtol=1e-13, atol=1e-14)
+    np.testing.assert_allclose(lse[..., 0], math.log(Nk), rtol=1e-15)
+    np.testing.assert_allclose(mass, L / Nk, rtol=1e-14)
+
+    a, scale = 1.5, 0.5
+    q = np.zeros((B, H, Mq, d), np.float32)
+    k = np.zeros((B, H, Nk, d), np.float32)
+    k[..., 0, 0] = 1.0
+    k[..., 1:, 1] = 1.0
+    q[..., 0] = a / scale
+    O, lse, _, _ = oracle_mod.attention(q, k, v, L, scale)
+    vv = v.astype(np.float64)
+    expect = (math.exp(a) * vv[:, :, :1] + vv[:, :, 1:].sum(2, keepdims=True)) / (math.exp(a) + Nk - 1)
+    np.testing.assert_allclose(O, np.broadcast_to(expect, O.shape), rtol=1e-13, atol=1e-14)
+    np.testing.assert_allclose(lse[..., 0], math.log(math.exp(a) + Nk - 1), rtol=1e-14)
+
+
+def test_attention_permutation_rows_and_accumulate(oracle_mod):
+    """Permuting the keys and values together (within the text block and within
+    the image block) leaves every output unchanged; permuting the values alone
+    changes O.  A row subset gives the same rows; accumulate adds w * A."""
+    rng = np.random.default_rng(5)
+    B, H, Mq, Nk, L, d = 2, 3, 7, 11, 4, 8
+    q = rng.standard_normal((B, H, Mq, d)).astype(np.float32)
+    k = rng.standard_normal((B, H, Nk, d)).astype(np.float32)
+    v = rng.standard_normal((B, H, Nk, d)).astype(np.float32)
+    O, lse, mass, A = oracle_mod.attention(q, k, v, L, 0.3)
+    perm = np.concatenate([rng.permutation(L), L + rng.permutation(Nk - L)])
+    O2, lse2, mass2, A2 = oracle_mod.attention(q, np.ascontiguousarray(k[:, :, perm]),
+                                               np.ascontiguousarray(v[:, :, perm]), L, 0.3)
+    np.testing.assert_allclose(O2, O, rtol=1e-12, atol=1e-13)
+    np.testing.assert_allclose(lse2, lse, rtol=1e-13)
+    np.testing.assert_allclose(mass2, mass, rtol=1e-12)
+    O3, _, _, _ = oracle_mod.attention(q, k, np.ascontiguousarray(v[:, :, perm]), L, 0.3)
+    assert np.abs(O3 - O).max() > 1e-3
+    rows = [3, Mq + 5, 0]
+    O4, _, _, A4 = oracle_mod.attention(q, k, v, L, 0.3, rows=rows)
+    for f in rows:
+        b, i = divmod(f, Mq)
+        np.testing.assert_array_equal(O4[b, :, i], O[b, :, i])
+        assert A4[b, i] == A[b, i]
+    A_in = rng.standard_normal((B, Mq)).astype(np.float32)
+    _, _, _, A5 = oracle_mod.attention(q, k, v, L, 0.3, weight=0.25, A_in=A_in)
+    np.testing.assert_allclose(A5, A_in + 0.25 * A.astype(np.float64), rtol=1e-6, atol=1e-7)
+
+
 def test_temporal_closed_forms(oracle_mod):
     """P2: h_t = c h_prev gives |c-1| |h| / (|h| + eps); h_prev = 0 gives |h_t|/eps."""
     rng = np.random.default_rng(1)
