@@ -368,6 +368,8 @@ def run_ours(args, world, rank, local, pg):
         result["edit"] = config_measure(torch, av, dev, stream, peaks, "edit")
         result["tiny"] = config_measure(torch, av, dev, stream, peaks, "tiny")
         result["batch_sweep"] = batch_sweep_measure(torch, av, dev, stream, peaks)
+        result["attention_forward"] = {
+            n: attention_measure(torch, av, dev, stream, peaks, n) for n in ("flux1024", "flux2048")}
     return result, tr
 
 
@@ -702,6 +704,59 @@ def lse_measure(torch, av, buf, tr, sets, nsets, stream, peaks):
     tf = flops / (ms * 1e-3) / 1e12
     return {"us": round(ms * 1e3, 3), "tflops": round(tf, 2),
             "frac_tensor": round(tf / peaks["bf16_tflops"], 4), "text_keys": tr.L,
+            "status": av.avits_device_status(stream)}
+
+
+def attention_measure(torch, av, dev, stream, peaks, name, nsets=5):
+    """The joint-attention forward with the spatial score (avits_attention_forward)
+    on the joint sequence of a configuration (queries = keys = text + image
+    tokens; Q, K, V bf16 rotated over nsets copies, more than L2), three ways:
+    with A and lse, with O only (the cost of the score is the difference), and
+    the separate spatial-score pass over the image rows that the forward makes
+    unnecessary."""
+    from paper_2608_17995_gb300.pipeline import to_device
+    from paper_2608_17995_gb300.workloads import make_transition, make_joint_attention
+    tr = make_transition(name)
+    q, v = make_joint_attention(tr)
+    B, H, Mq, d = q.shape
+    Nk = tr.Nk
+    sets = []
+    for i in range(nsets):
+        qd, kd, vd = (to_device(a, "bf16", dev) for a in (q, tr.k_all, v))
+        sets.append((qd, kd, vd, torch.empty_like(qd)))
+    A = torch.zeros(B, Mq, dtype=torch.float32, device=dev)
+    lse = torch.empty(B, H, Mq, 2, dtype=torch.float32, device=dev)
+    A_sp = torch.zeros(B, tr.M, dtype=torch.float32, device=dev)
+    ws = av.SpatialWorkspace(dev)
+
+    def fwd(with_score):
+        def fn():
+            for (qd, kd, vd, od) in sets:
+                av.avits_attention_forward(qd, kd, vd, tr.L, tr.softmax_scale, od,
+                                           lse=lse if with_score else None,
+                                           A=A if with_score else None, workspace=ws,
+                                           stream=stream)
+        return fn
+
+    def spatial():
+        for (qd, kd, _, _) in sets:
+            av.avits_score_spatial(qd[:, :, tr.L:tr.L + tr.M], kd, tr.L, tr.softmax_scale, A_sp,
+                                   workspace=ws, stream=stream)
+
+    reps = 20 if Mq <= 2048 else 5
+    ms_a = _graph_time_ms(torch, stream, fwd(True), reps) / nsets
+    ms_o = _graph_time_ms(torch, stream, fwd(False), reps) / nsets
+    ms_s = _graph_time_ms(torch, stream, spatial, reps) / nsets
+    flops = 4.0 * B * H * Mq * Nk * d
+    tf = flops / (ms_a * 1e-3) / 1e12
+    return {"shape": {"B": B, "H": H, "Mq": Mq, "Nk": Nk, "L": tr.L, "d": d},
+            "us": round(ms_a * 1e3, 3), "tflops": round(tf, 2),
+            "frac_tensor": round(tf / peaks["bf16_tflops"], 4),
+            "us_o_only": round(ms_o * 1e3, 3),
+            "tflops_o_only": round(flops / (ms_o * 1e-3) / 1e12, 2),
+            "score_cost_us": round((ms_a - ms_o) * 1e3, 3),
+            "separate_spatial_pass_us": round(ms_s * 1e3, 3),
+            "flops_per_call": flops,
             "status": av.avits_device_status(stream)}
 
 

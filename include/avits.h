@@ -14,6 +14,9 @@
  *     _keymask                  interleaved text keys given by a mask
  *     _lse                      from the model attention's logsumexp
  *     _noalloc                  without a caller workspace
+ *   avits_attention_forward   Eq. 4-5 + Eq. 3  the block's joint attention
+ *                             O = softmax(QK^T/sqrt d) V, with its logsumexp
+ *                             and the spatial score from the same softmax
  *   avits_score_temporal      Sec. 3.3.2      per-token relative step change
  *   avits_score_spatiotemporal  both scores in one call
  *   avits_score_temporal_var  Eq. 6-7         step variance over N_T snapshots
@@ -208,6 +211,51 @@ avits_status avits_score_spatial_keymask(const void* q_img, const void* k_all, a
                                          float softmax_scale, float weight, int accumulate,
                                          float* A, float* lse_opt, void* workspace,
                                          size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Joint-attention forward of a double-stream block (Eq. 4-5, Sec. 3.3.1) that
+ * also produces the spatial score of Eq. 3 from the same softmax.  The paper
+ * recomputes Q K^T after the block's attention only because fused attention
+ * kernels do not expose the weights; this call IS the block's attention and
+ * reads the text mass off it.  For batch b, head h and query row i:
+ *
+ *     l_ij   = softmax_scale * <q_bhi, k_bhj>                j = 0 .. Nk-1
+ *     o_bhi  = sum_j exp(l_ij) v_bhj / sum_j exp(l_ij)
+ *     mass   = sum_{j<L} exp(l_ij) / sum_{j<Nk} exp(l_ij)    (text keys first)
+ *     A[b,i] = (accumulate ? A[b,i] : 0) + weight * (1/H) * sum_h mass
+ *
+ * q : [B,H,Mq,d] bf16, the joint queries [Q_txt || Q_img] of Eq. 4 (any rows:
+ *     text and image rows alike; A and lse are given for every row).
+ * k, v : [B,H,Nk,d] bf16, the joint keys / values, the L text keys FIRST.
+ * o : [B,H,Mq,d] bf16 output (must not overlap q, k, v).
+ * q_str, k_str, v_str, o_str : element strides (batch, head, row) of each
+ *     tensor as an array of 3 int64, or NULL for contiguous [B,H,rows,d]; the
+ *     d axis is contiguous.  Bases 16-byte aligned, strides multiples of 8
+ *     elements ([B,N,H,d] views of a model's projections qualify).
+ * d in {64, 128}; 0 <= L <= Nk; softmax_scale > 0 (1/sqrt(d)).
+ * lse_opt : NULL or [B,H,Mq,2] fp32: natural-log logsumexp of the row over
+ *     all keys and over the text keys (-inf when L = 0).
+ * A : NULL (no score; workspace may then be NULL) or [B,Mq] fp32, written
+ *     (accumulate = 0) or added to; H <= 255 when A is given.
+ * workspace/ws_bytes : when A is given, avits_attention_forward_workspace()
+ *     bytes, 8-byte aligned, ZERO-FILLED before first use; every call that
+ *     completes leaves it zero, so it is reused as is (re-zero it after
+ *     AVITS_ERR_TIMEOUT).  One workspace per concurrently running call.
+ * Precision: P = softmax numerators enter the P V product rounded to bf16
+ *     (fp32 accumulation, fp32 row sums), O is rounded to bf16 once.
+ * Other dtypes or d values return AVITS_ERR_UNSUPPORTED; one kernel launch.
+ * ---------------------------------------------------------------------- */
+avits_status avits_attention_forward(const void* q, const void* k, const void* v, avits_dtype dt,
+                                     int B, int H, int Mq, int Nk, int L, int d,
+                                     const int64_t* q_str, const int64_t* k_str,
+                                     const int64_t* v_str, const int64_t* o_str,
+                                     float softmax_scale, void* o, float* lse_opt, float weight,
+                                     int accumulate, float* A, void* workspace, size_t ws_bytes,
+                                     void* stream);
+
+/* Workspace bytes of avits_attention_forward with a score output (0 for
+ * invalid sizes). */
+size_t avits_attention_forward_workspace(int B, int H, int Mq);
 
 /* ------------------------------------------------------------------------
  * Temporal importance.  Sec. 3.3.2 scores a token by how much its feature

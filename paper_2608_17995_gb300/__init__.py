@@ -85,6 +85,9 @@ def lib():
         "avits_score_spatial_lse": [vp, vp, i32, i32, i32, i32, i32, i32, i64, i64, i64, i64,
                                     i64, i64, vp, f32, f32, i32, vp, vp, vp, sz, vp],
         "avits_score_temporal": [vp, vp, i32, i32, i32, i32, f32, vp, vp],
+        "avits_attention_forward": [vp, vp, vp, i32, i32, i32, i32, i32, i32, i32, vp, vp, vp, vp,
+                                    f32, vp, vp, f32, i32, vp, vp, sz, vp],
+        "avits_attention_forward_workspace": [i32, i32, i32],
         "avits_score_spatiotemporal": [vp, vp, i32, i32, i32, i32, i32, i32, i32, i64, i64, i64,
                                        i64, i64, i64, f32, f32, i32, vp, vp, vp, sz, vp, vp, i32,
                                        f32, vp, vp],
@@ -112,7 +115,7 @@ def lib():
         fn.argtypes = args
         fn.restype = ctypes.c_int
     for name in ("avits_score_spatial_workspace", "avits_merge_final_workspace",
-                 "avits_score_spatial_noalloc_limit"):
+                 "avits_score_spatial_noalloc_limit", "avits_attention_forward_workspace"):
         getattr(L, name).restype = ctypes.c_size_t
     for name in ("avits_status_string", "avits_last_error_string", "avits_version",
                  "avits_score_spatial_noalloc_error"):
@@ -317,6 +320,51 @@ def avits_score_spatiotemporal(q_img, k_all, L: int, softmax_scale: float, A, h_
         _stream(stream))
     _check("avits_score_spatiotemporal", rc)
     return A, V
+
+
+def avits_attention_forward_workspace(B: int, H: int, Mq: int) -> int:
+    return int(lib().avits_attention_forward_workspace(B, H, Mq))
+
+
+def _strides3(t):
+    arr = (ctypes.c_int64 * 3)(t.stride(0), t.stride(1), t.stride(2))
+    return arr
+
+
+def avits_attention_forward(q, k, v, L: int, softmax_scale: float, o, lse=None, A=None,
+                            weight: float = 1.0, accumulate: bool = False,
+                            workspace: Optional[SpatialWorkspace] = None, stream=None):
+    """Eq. 4-5 + Eq. 3: the joint-attention forward O = softmax(scale Q K^T) V
+    of a double-stream block (q [B,H,Mq,d], k / v [B,H,Nk,d], bf16, any
+    strides with d contiguous, the L text keys first) into o [B,H,Mq,d]
+    bf16, with lse [B,H,Mq,2] (all keys, text keys) and the spatial score A
+    [B,Mq] (written or accumulated) when given."""
+    B, H, Mq, d = q.shape
+    Nk = k.shape[2]
+    if tuple(k.shape) != (B, H, Nk, d) or tuple(v.shape) != (B, H, Nk, d) or \
+            tuple(o.shape) != (B, H, Mq, d):
+        raise ValueError("q / k / v / o shapes disagree")
+    for t in (q, k, v, o):
+        if t.stride(3) != 1:
+            raise ValueError("the head-dim axis must be contiguous")
+    dt = _dtype_code(q)
+    if _dtype_code(k) != dt or _dtype_code(v) != dt or _dtype_code(o) != dt:
+        raise TypeError("q, k, v and o dtypes differ")
+    wbuf, wbytes = None, 0
+    if A is not None:
+        need = avits_attention_forward_workspace(B, H, Mq)
+        if workspace is None:
+            key = ("attn", q.device.index,
+                   _torch().cuda.current_stream().cuda_stream if stream is None else _stream(stream))
+            workspace = _default_ws.setdefault(key, SpatialWorkspace(q.device))
+        wbuf, wbytes = workspace.get(need)
+    qs, ks, vs, os_ = _strides3(q), _strides3(k), _strides3(v), _strides3(o)
+    rc = lib().avits_attention_forward(
+        _ptr(q), _ptr(k), _ptr(v), dt, B, H, Mq, Nk, L, d, qs, ks, vs, os_,
+        float(softmax_scale), _ptr(o), _ptr(lse), float(weight), 1 if accumulate else 0,
+        _ptr(A), _ptr(wbuf), wbytes, _stream(stream))
+    _check("avits_attention_forward", rc)
+    return o
 
 
 def avits_score_temporal(h_t, h_prev, V, eps: float = 1e-6, stream=None):

@@ -161,6 +161,55 @@ avits_status avits_score_spatial_keymask(const void* q_img, const void* k_all, a
   return cuda_status(launch_spatial_simt(a, s));
 }
 
+size_t avits_attention_forward_workspace(int B, int H, int Mq) {
+  if (B <= 0 || H <= 0 || Mq <= 0) return 0;
+  return attention_tc_workspace(B, H, Mq);
+}
+
+avits_status avits_attention_forward(const void* q, const void* k, const void* v, avits_dtype dt,
+                                     int B, int H, int Mq, int Nk, int L, int d,
+                                     const int64_t* q_str, const int64_t* k_str,
+                                     const int64_t* v_str, const int64_t* o_str,
+                                     float softmax_scale, void* o, float* lse_opt, float weight,
+                                     int accumulate, float* A, void* workspace, size_t ws_bytes,
+                                     void* stream) {
+  AVITS_RANGE();
+  if (!q || !k || !v || !o || !valid_dtype(dt)) return AVITS_ERR_INVALID_ARG;
+  if (B <= 0 || H <= 0 || Mq <= 0 || Nk <= 0 || d <= 0 || L < 0 || L > Nk)
+    return AVITS_ERR_INVALID_ARG;
+  if (!(softmax_scale > 0.f) || !(softmax_scale < 3.0e38f)) return AVITS_ERR_INVALID_ARG;
+  AttnArgs a{};
+  a.q = q; a.k = k; a.v = v; a.o = o;
+  a.B = B; a.H = H; a.Mq = Mq; a.Nk = Nk; a.L = L; a.d = d;
+  const int64_t* given[4] = {q_str, k_str, v_str, o_str};
+  for (int i = 0; i < 4; ++i) {
+    const int64_t rows = (i == 1 || i == 2) ? Nk : Mq;
+    if (given[i]) {
+      for (int j = 0; j < 3; ++j) a.str[i][j] = given[i][j];
+      if (a.str[i][2] < d || a.str[i][1] < 0 || a.str[i][0] < 0) return AVITS_ERR_INVALID_ARG;
+    } else {
+      a.str[i][2] = d;
+      a.str[i][1] = rows * d;
+      a.str[i][0] = (int64_t)H * rows * d;
+    }
+  }
+  a.scale = softmax_scale;
+  a.weight = weight;
+  a.accumulate = accumulate ? 1 : 0;
+  a.A = A;
+  a.lse = lse_opt;
+  a.ws = workspace;
+  a.status = status_word();
+  if (A && (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 7u) ||
+            ws_bytes < attention_tc_workspace(B, H, Mq)))
+    return AVITS_ERR_INVALID_ARG;
+  if (dt != AVITS_BF16) return AVITS_ERR_UNSUPPORTED;
+  if (A && H > 255) return AVITS_ERR_UNSUPPORTED;   // the head count of the fixed-point sum
+  if ((long long)B * H * ((Mq + 255) / 256) >= (1ll << 31)) return AVITS_ERR_UNSUPPORTED;
+  if (!attention_tc_layout_ok(a)) return AVITS_ERR_UNSUPPORTED;
+  return cuda_status(launch_attention_tc(a, num_sms_current(), static_cast<cudaStream_t>(stream)));
+}
+
 avits_status avits_score_temporal(const void* h_t, const void* h_prev, avits_dtype dt, int B,
                                   int N, int D, float eps, float* V, void* stream) {
   AVITS_RANGE();

@@ -1,0 +1,633 @@
+// attention_tc.cu — the joint-attention forward of a double-stream block
+// (Eq. 4-5, Sec. 3.3.1) on the sm_103a tensor cores, with the spatial score
+// of Eq. 3 read off the same softmax.
+//
+// For batch b, head h and query row i of the joint sequence [C; Z]:
+//   O_i      = sum_j softmax_j(scale * q_i . k_j) v_j        (all Nk keys)
+//   lse_i    = log sum_j exp(scale * q_i . k_j), over all keys and over the
+//              text keys (the first L)
+//   A_i     (+)= weight * mean_h exp(lse_txt_i - lse_all_i)  (Eq. 5, Eq. 3)
+// The text mass Eq. 5 extracts is a by-product of the softmax the block
+// computes anyway: the only extra work is one running sum per row.
+//
+// Work decomposition (persistent, one CTA per SM): unit = (b, h, 256 query
+// rows = two 128-row tiles); CTA c takes units c, c + grid, ...  Each unit
+// runs over all key tiles (128 keys), so O and the row statistics stay in
+// the CTA and no partial results cross CTAs (except Eq. 3's head sum).
+//
+// Tensor memory (512 columns): S_t / P_t of query tile t at columns
+// [128t, 128t + 128), O_t at [256 + Dt, 256 + D(t+1)).  P_t (bf16 pairs)
+// overwrites the first 64 columns of S_t, each 16-column block after the
+// softmax has read the 32 S columns it replaces.
+//
+// Roles (12 warps):
+//   warp 0       TMA producer: Q tile 0, K_0, Q tile 1, V_0, then K_j, V_j
+//                through a ring of 128-key tiles (128-byte swizzle).
+//   warps 1, 2   MMA issuers of query tile 0 / 1 (warp 1 owns tensor
+//                memory): per key tile S_t = Q_t K_j^T (tcgen05.mma, both
+//                operands K-major in shared memory), then, once the softmax
+//                has written P_t, O_t += P_t V_j (A = P_t from tensor memory,
+//                B = V_j as an MN-major shared-memory operand, no transpose
+//                copy).  S_t of the next key tile overwrites P_t, so it is
+//                issued when that PV product has completed; the other tile's
+//                issuer keeps the tensor pipe busy meanwhile.
+//   warp 3       no role.
+//   warps 4-7    softmax and epilogue of query tile 0, warps 8-11 of tile 1:
+//                one row per thread (TMEM lane), two passes over the 128 S
+//                columns of an item (row maximum, then exponentials, sums and
+//                P).  The running maximum is raised only when a key tile's
+//                maximum exceeds it by more than 2^8 (P <= 256 otherwise, no
+//                loss in bf16 or the fp32 accumulator); then l and O are
+//                rescaled in place.  The epilogue divides O by the row sum,
+//                stages it in shared memory in the TMA's swizzled layout and
+//                stores it with one bulk tensor copy per 64 columns.
+// Every wait is bounded (avits_common.cuh); after a timeout every role skips
+// its remaining work, drains what it issued and the CTA releases tensor
+// memory and exits.
+#include <cuda.h>
+
+#include "avits_common.cuh"
+#include "avits_internal.h"
+#include "tc_common.cuh"
+
+namespace avits {
+namespace {
+
+using namespace tc;
+
+constexpr int kBM = 128;            // query rows per tile (= TMEM lanes)
+constexpr int kBN = 128;            // keys per tile
+constexpr int kQTiles = 2;          // query tiles per unit
+constexpr int kUnitRows = kBM * kQTiles;
+constexpr int kThreads = 12 * 32;
+constexpr int kTmemCols = 512;
+constexpr float kTau = 8.f;         // lazy rescale threshold (log2 units)
+constexpr uint32_t kIdescS = idesc_bf16(kBM, kBN, false);
+
+template <int D>
+struct Cfg {
+  static constexpr int kCB = D / 64;                   // 128-byte column blocks per row
+  static constexpr int kTileBytes = kCB * kBM * 128;   // one 128-row bf16 tile
+  static constexpr int kStages = (D == 128) ? 3 : 6;   // K / V ring
+  static constexpr int kQBytes = kQTiles * kTileBytes;
+  static constexpr int kKVBytes = kStages * kTileBytes;
+  static constexpr int kOBytes = kQTiles * kTileBytes; // O staging, one tile each
+  static constexpr uint32_t kIdescPV = idesc_bf16(kBM, D, true);
+};
+constexpr int kMaxStages = 6;
+
+struct Bars {
+  uint64_t q_full[kQTiles], q_empty[kQTiles];
+  uint64_t kv_full[kMaxStages], kv_empty[kMaxStages];
+  uint64_t s_full[kQTiles], p_full[kQTiles], pv_done[kQTiles];
+  uint64_t o_full[kQTiles], o_empty[kQTiles], drain[kQTiles];
+  uint32_t tmem_base;
+  int abort;
+};
+
+template <int D>
+constexpr int smem_bytes() {
+  return Cfg<D>::kQBytes + Cfg<D>::kKVBytes + Cfg<D>::kOBytes + (int)sizeof(Bars) + 1024;
+}
+
+struct AttnParams {
+  int B, H, Mq, Nk, L;
+  int n_qp, n_kt, n_units;
+  float c_log2, weight;
+  int accumulate;
+  float* A;                   // [B,Mq] or NULL
+  float* lse;                 // [B,H,Mq,2] or NULL
+  unsigned long long* acc;    // [B][n_qp * 256] head-sum words (A != NULL)
+  int rows_pad;
+  unsigned int* status;
+};
+
+// WG-wide AND of v over the `count` threads of named barrier `id`.
+__device__ __forceinline__ bool bar_and(int id, int count, bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.and.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)v), "r"(id), "r"(count)
+      : "memory");
+  return r != 0;
+}
+
+__device__ __forceinline__ void wait_ld2(uint32_t (&a)[32], uint32_t (&b)[32]) {
+  tmem_wait32(a);
+  tmem_wait32(b);   // already complete; ties b's registers to the wait
+}
+
+// Row maximum of 32 S columns whose first key is col0; keys >= Nk are left
+// out (kFull: all 32 are valid).
+template <bool kFull>
+__device__ __forceinline__ float chunk_max(const uint32_t (&r)[32], int col0, int Nk) {
+  float v[32];
+#pragma unroll
+  for (int e = 0; e < 32; ++e) v[e] = __uint_as_float(r[e]);
+  if (!kFull) {
+#pragma unroll
+    for (int e = 0; e < 32; ++e)
+      if (col0 + e >= Nk) v[e] = -INFINITY;
+  }
+  float t[11];
+#pragma unroll
+  for (int g = 0; g < 10; ++g) t[g] = max3(v[3 * g], v[3 * g + 1], v[3 * g + 2]);
+  t[10] = fmaxf(v[30], v[31]);
+  const float u0 = max3(t[0], t[1], t[2]), u1 = max3(t[3], t[4], t[5]);
+  const float u2 = max3(t[6], t[7], t[8]);
+  return fmaxf(max3(u0, u1, u2), fmaxf(t[9], t[10]));
+}
+
+// Exponentials of 32 S columns (first key col0) against the running maximum
+// m: their fp32 sum (all keys, text keys) and the bf16 P words for tensor
+// memory.  kKind: 0 = valid image keys, 1 = valid text keys, 2 = general
+// (keys beyond Nk give 0, text keys counted one by one).
+template <int kKind>
+__device__ __forceinline__ void chunk_exp(const uint32_t (&r)[32], int col0, int Nk, int L,
+                                          float c, float m, float& la, float& lt,
+                                          uint32_t (&w)[16]) {
+  const float nm = -m;
+  float p[32];
+#pragma unroll
+  for (int e = 0; e < 32; e += 2) {
+    float x0, x1;
+    ffma2(__uint_as_float(r[e]), __uint_as_float(r[e + 1]), c, nm, x0, x1);
+    p[e] = ex2(x0);
+    p[e + 1] = ex2(x1);
+  }
+  if (kKind == 2) {
+#pragma unroll
+    for (int e = 0; e < 32; ++e)
+      if (col0 + e >= Nk) p[e] = 0.f;
+  }
+  float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+  for (int e = 0; e < 32; e += 4) {
+    fadd2(s0, s1, p[e], p[e + 1]);
+    fadd2(s2, s3, p[e + 2], p[e + 3]);
+  }
+  fadd2(s0, s1, s2, s3);
+  const float cs = s0 + s1;
+  la += cs;
+  if (kKind == 1) {
+    lt += cs;
+  } else if (kKind == 2 && col0 < L) {
+    float ts = 0.f;
+#pragma unroll
+    for (int e = 0; e < 32; ++e) ts += (col0 + e < L) ? p[e] : 0.f;
+    lt += ts;
+  }
+#pragma unroll
+  for (int e = 0; e < 16; ++e) w[e] = pack_bf16x2(p[2 * e], p[2 * e + 1]);
+}
+
+// Kind of the 32 keys starting at col0 (uniform over the warp).
+__device__ __forceinline__ int chunk_kind(int col0, int Nk, int L) {
+  if (col0 + 32 <= Nk) {
+    if (col0 + 32 <= L) return 1;
+    if (col0 >= L) return 0;
+  }
+  return 2;
+}
+
+__device__ __forceinline__ void exp_by_kind(int kind, const uint32_t (&r)[32], int col0, int Nk,
+                                            int L, float c, float m, float& la, float& lt,
+                                            uint32_t (&w)[16]) {
+  if (kind == 0)
+    chunk_exp<0>(r, col0, Nk, L, c, m, la, lt, w);
+  else if (kind == 1)
+    chunk_exp<1>(r, col0, Nk, L, c, m, la, lt, w);
+  else
+    chunk_exp<2>(r, col0, Nk, L, c, m, la, lt, w);
+}
+
+// O_t row *= f (D fp32 columns at tO).
+template <int D>
+__device__ __forceinline__ void rescale_o(uint32_t tO, float f) {
+#pragma unroll 1
+  for (int k = 0; k < D / 32; ++k) {
+    uint32_t r[32];
+    tmem_ld32(tO + 32 * k, r);
+    tmem_wait32(r);
+#pragma unroll
+    for (int e = 0; e < 32; e += 2) {
+      float a0 = __uint_as_float(r[e]), a1 = __uint_as_float(r[e + 1]);
+      fmul2(a0, a1, f);
+      r[e] = __float_as_uint(a0);
+      r[e + 1] = __float_as_uint(a1);
+    }
+    tmem_st32(tO + 32 * k, r);
+  }
+}
+
+struct RowState {
+  float m, la, lt;
+};
+
+// One key tile of one row: S at tS (128 fp32 columns), P written to the
+// first 64 columns, the running statistics updated, O rescaled when the
+// maximum moves.  first: the row's first key tile of the unit (O holds no
+// sum yet).
+template <int D>
+__device__ __forceinline__ void softmax_item(uint32_t tS, uint32_t tO, int key0, int Nk, int L,
+                                             float c, bool first, RowState& st) {
+  uint32_t ra[32], rb[32];
+  const bool full = key0 + kBN <= Nk;
+  // pass 1: the tile's row maximum
+  tmem_ld32(tS, ra);
+  tmem_ld32(tS + 32, rb);
+  wait_ld2(ra, rb);
+  float mx = full ? fmaxf(chunk_max<true>(ra, 0, 0), chunk_max<true>(rb, 0, 0))
+                  : fmaxf(chunk_max<false>(ra, key0, Nk), chunk_max<false>(rb, key0 + 32, Nk));
+  tmem_ld32(tS + 64, ra);
+  tmem_ld32(tS + 96, rb);
+  wait_ld2(ra, rb);
+  mx = full ? fmaxf(mx, fmaxf(chunk_max<true>(ra, 0, 0), chunk_max<true>(rb, 0, 0)))
+            : fmaxf(mx, fmaxf(chunk_max<false>(ra, key0 + 64, Nk),
+                              chunk_max<false>(rb, key0 + 96, Nk)));
+  const float mt = mx * c;
+  const bool up = mt > st.m + kTau;   // the row's first tile, or a logit 2^8 above its maximum
+  float f = 1.f;
+  if (up) {
+    f = ex2(st.m - mt);
+    st.la *= f;
+    st.lt *= f;
+    st.m = mt;
+  }
+  // tcgen05.ld / st are warp-collective: the warp rescales its O rows
+  // together when any of them moved (f = 1 leaves a row unchanged)
+  if (!first && __any_sync(0xffffffffu, up)) rescale_o<D>(tO, f);
+  // pass 2: exponentials, sums and P, 32 columns at a time; P block k
+  // (columns [16k, 16k + 16)) replaces S columns already read
+  uint32_t w[16];
+  tmem_ld32(tS, ra);
+  tmem_wait32(ra);
+  tmem_ld32(tS + 32, rb);
+  exp_by_kind(chunk_kind(key0, Nk, L), ra, key0, Nk, L, c, st.m, st.la, st.lt, w);
+  tmem_st16(tS, w);
+  tmem_wait32(rb);
+  tmem_ld32(tS + 64, ra);
+  exp_by_kind(chunk_kind(key0 + 32, Nk, L), rb, key0 + 32, Nk, L, c, st.m, st.la, st.lt, w);
+  tmem_st16(tS + 16, w);
+  tmem_wait32(ra);
+  tmem_ld32(tS + 96, rb);
+  exp_by_kind(chunk_kind(key0 + 64, Nk, L), ra, key0 + 64, Nk, L, c, st.m, st.la, st.lt, w);
+  tmem_st16(tS + 32, w);
+  tmem_wait32(rb);
+  exp_by_kind(chunk_kind(key0 + 96, Nk, L), rb, key0 + 96, Nk, L, c, st.m, st.la, st.lt, w);
+  tmem_st16(tS + 48, w);
+  tmem_wait_st();
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                    const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
+                    const AttnParams p) {
+  using C = Cfg<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sQ = smem;
+  uint8_t* sKV = sQ + C::kQBytes;
+  uint8_t* sO = sKV + C::kKVBytes;
+  Bars* bars = reinterpret_cast<Bars*>(sO + C::kOBytes);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n_my = (p.n_units - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
+  if (n_my <= 0) return;   // block-uniform
+
+  if (threadIdx.x == 0) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQ)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmO)) : "memory");
+    for (int t = 0; t < kQTiles; ++t) {
+      mbar_init(&bars->q_full[t], 1);
+      mbar_init(&bars->q_empty[t], 1);
+      mbar_init(&bars->s_full[t], 1);
+      mbar_init(&bars->p_full[t], 4);     // the tile's 4 softmax warps
+      mbar_init(&bars->pv_done[t], 1);
+      mbar_init(&bars->o_full[t], 1);
+      mbar_init(&bars->o_empty[t], 4);
+      mbar_init(&bars->drain[t], 1);
+    }
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(&bars->kv_full[s], 1);
+      mbar_init(&bars->kv_empty[s], kQTiles);   // one commit per issuer
+    }
+    bars->abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    fence_async_shared();
+  }
+  // Q, K and V may come from the kernel before this one on the stream
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  if (warp == 1) tmem_alloc(&bars->tmem_base, kTmemCols);
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = bars->tmem_base;
+  volatile int* abort_flag = &bars->abort;
+  if (threadIdx.x == 96) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+  auto unit_coords = [&](int u, int& b, int& h, int& qp) {
+    const int bh = u / p.n_qp;
+    qp = u - bh * p.n_qp;
+    b = bh / p.H;
+    h = bh - b * p.H;
+  };
+
+  if (warp == 0) {
+    // ------------------------------------------------------ TMA producer --
+    if (lane == 0) {
+      bool ok = true;
+      int li = 0;        // ring loads issued (K and V tiles)
+      int q_armed = 0;   // Q tiles of the current unit issued
+      int ui = 0;
+      for (; ui < n_my && ok; ++ui) {
+        int b, h, qp;
+        unit_coords((int)blockIdx.x + ui * (int)gridDim.x, b, h, qp);
+        q_armed = 0;
+        auto load_q = [&](int t) {
+          if (ui > 0) ok = mbar_wait_bounded(&bars->q_empty[t], (uint32_t)((ui - 1) & 1), abort_flag, p.status);
+          if (!ok) return;
+          mbar_arrive_expect_tx(&bars->q_full[t], C::kTileBytes);
+          for (int cb = 0; cb < C::kCB; ++cb)
+            tma_load_4d(sQ + t * C::kTileBytes + cb * (kBM * 128), &tmQ, cb * 64,
+                        qp * kUnitRows + t * kBM, h, b, &bars->q_full[t]);
+          ++q_armed;
+        };
+        auto load_kv = [&](const CUtensorMap* map, int kt) {
+          const int stage = li % C::kStages;
+          const uint32_t ph = (uint32_t)((li / C::kStages) & 1);
+          ok = mbar_wait_bounded(&bars->kv_empty[stage], ph ^ 1u, abort_flag, p.status);
+          if (!ok) return;
+          mbar_arrive_expect_tx(&bars->kv_full[stage], C::kTileBytes);
+          for (int cb = 0; cb < C::kCB; ++cb)
+            tma_load_4d(sKV + stage * C::kTileBytes + cb * (kBM * 128), map, cb * 64, kt * kBN, h,
+                        b, &bars->kv_full[stage]);
+          ++li;
+        };
+        load_q(0);
+        if (ok) load_kv(&tmK, 0);
+        if (ok) load_q(1);
+        for (int j = 0; j < p.n_kt && ok; ++j) {
+          load_kv(&tmV, j);
+          if (ok && j + 1 < p.n_kt) load_kv(&tmK, j + 1);
+        }
+      }
+      if (!ok) {
+        // drain the copies still in flight: the Q tiles of the last unit
+        // started, then the last load of every ring stage
+        const int ul = ui - 1;
+        for (int t = 0; t < q_armed; ++t)
+          mbar_wait_bounded(&bars->q_full[t], (uint32_t)(ul & 1), nullptr, p.status);
+        for (int s = 0; s < C::kStages; ++s) {
+          const int armed = li - s;   // loads issued on stage s: li - s > 0
+          if (armed > 0) {
+            const int last = (armed - 1) / C::kStages;
+            mbar_wait_bounded(&bars->kv_full[s], (uint32_t)(last & 1), nullptr, p.status);
+          }
+        }
+      }
+    }
+  } else if (warp == 1 || warp == 2) {
+    // -------------------------------------------------------- MMA issuers --
+    const int t = warp - 1;
+    if (lane == 0) {
+      bool ok = true;
+      int gi = 0;   // key tiles processed by this CTA (all units)
+      const uint32_t a_lo = sw128_desc_lo(sQ + t * C::kTileBytes);
+      const uint32_t kv_lo0 = sw128_desc_lo(sKV);
+      const uint32_t v_lo0 = sw128_mn_desc_lo(sKV, kBM * 128);
+      const uint32_t d_hi = sw128_desc_hi();
+      const uint32_t tS = tmem + (uint32_t)(t * kBN);
+      const uint32_t tO = tmem + (uint32_t)(2 * kBN + t * D);
+      for (int ui = 0; ui < n_my && ok; ++ui) {
+        for (int j = 0; j < p.n_kt && ok; ++j, ++gi) {
+          // S_t = Q_t K_j^T
+          const int lk = 2 * gi, lv = 2 * gi + 1;
+          const int sk = lk % C::kStages, sv = lv % C::kStages;
+          ok = mbar_wait_bounded(&bars->kv_full[sk], (uint32_t)((lk / C::kStages) & 1), abort_flag, p.status);
+          if (ok && j == 0)
+            ok = mbar_wait_bounded(&bars->q_full[t], (uint32_t)(ui & 1), abort_flag, p.status);
+          // P_t of the previous key tile has been read by its PV product
+          if (ok && gi > 0)
+            ok = mbar_wait_bounded(&bars->pv_done[t], (uint32_t)((gi - 1) & 1), abort_flag, p.status);
+          if (!ok) break;
+          fence_after();
+          const uint32_t k_lo = kv_lo0 + (uint32_t)((sk * C::kTileBytes) >> 4);
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t off = (uint32_t)(((kk >> 2) * (kBM * 128) + (kk & 3) * 32) >> 4);
+            mma_ss(tS, a_lo + off, k_lo + off, d_hi, kIdescS, kk > 0 ? 1u : 0u);
+          }
+          mma_commit(&bars->s_full[t]);
+          mma_commit(&bars->kv_empty[sk]);
+          if (j == p.n_kt - 1) mma_commit(&bars->q_empty[t]);
+          // O_t += P_t V_j
+          ok = mbar_wait_bounded(&bars->p_full[t], (uint32_t)(gi & 1), abort_flag, p.status);
+          if (ok)
+            ok = mbar_wait_bounded(&bars->kv_full[sv], (uint32_t)((lv / C::kStages) & 1), abort_flag, p.status);
+          if (ok && j == 0 && ui > 0)   // the epilogue has read the previous unit's O_t
+            ok = mbar_wait_bounded(&bars->o_empty[t], (uint32_t)((ui - 1) & 1), abort_flag, p.status);
+          if (!ok) break;
+          fence_after();
+          const uint32_t v_lo = v_lo0 + (uint32_t)((sv * C::kTileBytes) >> 4);
+#pragma unroll
+          for (int kk = 0; kk < kBN / 16; ++kk)   // 16 keys: 8 P columns, 16 V rows
+            mma_ts(tO, tS + (uint32_t)(kk * 8), v_lo + (uint32_t)((kk * 16 * 128) >> 4), d_hi,
+                   C::kIdescPV, (j > 0 || kk > 0) ? 1u : 0u);
+          mma_commit(&bars->pv_done[t]);
+          mma_commit(&bars->kv_empty[sv]);
+          if (j == p.n_kt - 1) mma_commit(&bars->o_full[t]);
+        }
+      }
+      // all issued MMAs complete before tensor memory is released
+      mma_commit(&bars->drain[t]);
+      mbar_wait_bounded(&bars->drain[t], 0, nullptr, p.status);
+    }
+  } else if (warp >= 4) {
+    // --------------------------------------------- softmax and epilogue --
+    const int t = (warp - 4) >> 2;
+    const int quad = warp & 3;             // TMEM lane quadrant this warp may access
+    const int rowt = quad * 32 + lane;     // row within the tile = TMEM lane
+    const int bar_id = 1 + t;              // named barrier of the tile's 128 threads
+    const bool leader = (quad == 0 && lane == 0);
+    const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
+    const uint32_t tS = tmem + lane_off + (uint32_t)(t * kBN);
+    const uint32_t tO = tmem + lane_off + (uint32_t)(2 * kBN + t * D);
+    uint8_t* stg = sO + t * C::kTileBytes;
+    bool ok = true;
+    int gi = 0;
+    for (int ui = 0; ui < n_my; ++ui) {
+      int b, h, qp;
+      unit_coords((int)blockIdx.x + ui * (int)gridDim.x, b, h, qp);
+      RowState st{-INFINITY, 0.f, 0.f};
+      for (int j = 0; j < p.n_kt; ++j, ++gi) {
+        ok = ok && (*abort_flag == 0) &&
+             mbar_wait_bounded(&bars->s_full[t], (uint32_t)(gi & 1), abort_flag, p.status);
+        ok = __all_sync(0xffffffffu, ok);   // tcgen05.ld / st are warp-collective
+        if (ok) {
+          fence_after();
+          softmax_item<D>(tS, tO, j * kBN, p.Nk, p.L, p.c_log2, j == 0, st);
+          fence_before();
+        }
+        __syncwarp();
+        if (ok && lane == 0) mbar_arrive(&bars->p_full[t]);
+      }
+      // ---- epilogue: O / l -> bf16 -> swizzled staging -> TMA store
+      ok = ok && (*abort_flag == 0) &&
+           mbar_wait_bounded(&bars->o_full[t], (uint32_t)(ui & 1), abort_flag, p.status);
+      ok = __all_sync(0xffffffffu, ok);
+      if (leader) bulk_wait_read();   // the previous unit's store has read the staging tile
+      bar_sync(bar_id, 128);
+      if (ok) {
+        fence_after();
+        const float inv = 1.f / st.la;
+#pragma unroll 1
+        for (int k = 0; k < D / 32; ++k) {
+          uint32_t r[32];
+          tmem_ld32(tO + 32 * k, r);
+          tmem_wait32(r);
+          uint32_t w[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e)
+            w[e] = pack_bf16x2(__uint_as_float(r[2 * e]) * inv, __uint_as_float(r[2 * e + 1]) * inv);
+          // columns [32k, 32k + 32): block cb, 16-byte chunks jj .. jj + 3 of
+          // the row, each at chunk (jj ^ row) of the 128-byte swizzle
+          const int cb = (32 * k) >> 6;
+          const int jj0 = ((32 * k) & 63) >> 3;
+          uint8_t* rowp = stg + cb * (kBM * 128) + rowt * 128;
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            *reinterpret_cast<uint4*>(rowp + (((jj0 + q) ^ (rowt & 7)) << 4)) =
+                make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+        }
+        fence_before();
+      }
+      __syncwarp();
+      if (ok && lane == 0) mbar_arrive(&bars->o_empty[t]);
+      const int row = qp * kUnitRows + t * kBM + rowt;
+      if (ok && row < p.Mq) {
+        const float ln2 = 0.69314718055994530942f;
+        if (p.lse) {
+          float* lp = p.lse + (((long long)b * p.H + h) * p.Mq + row) * 2;
+          lp[0] = (st.m + log2f(st.la)) * ln2;
+          lp[1] = st.lt > 0.f ? (st.m + log2f(st.lt)) * ln2 : -INFINITY;
+        }
+        if (p.A)
+          head_sum_add(p.acc + (long long)b * p.rows_pad + row, p.H, st.lt / st.la, p.weight,
+                       p.accumulate, p.A + (long long)b * p.Mq + row);
+      }
+      fence_async_shared();
+      const bool all_ok = bar_and(bar_id, 128, ok);
+      if (all_ok && leader && qp * kUnitRows + t * kBM < p.Mq) {   // a tile past the end stores nothing
+        for (int cb = 0; cb < C::kCB; ++cb)
+          tma_store_4d(&tmO, stg + cb * (kBM * 128), cb * 64, qp * kUnitRows + t * kBM, h, b);
+        bulk_commit();
+      }
+    }
+    if (leader) bulk_wait_all();
+  }
+
+  fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+struct Plan {
+  int n_qp, n_kt, n_units, grid;
+  size_t acc_bytes;
+};
+
+Plan make_plan(int B, int H, int Mq, int Nk, int num_sms) {
+  Plan pl{};
+  pl.n_qp = (Mq + kUnitRows - 1) / kUnitRows;
+  pl.n_kt = (Nk + kBN - 1) / kBN;
+  pl.n_units = B * H * pl.n_qp;
+  const int sms = num_sms > 0 ? num_sms : 1;
+  pl.grid = pl.n_units < sms ? pl.n_units : sms;
+  pl.acc_bytes = (sizeof(unsigned long long) * (size_t)B * pl.n_qp * kUnitRows + 255) &
+                 ~static_cast<size_t>(255);
+  return pl;
+}
+
+template <auto Kernel, int D>
+cudaError_t smem_attrs() {
+  cudaError_t e = cudaFuncSetAttribute(Kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                       cudaSharedmemCarveoutMaxShared);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(Kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<D>());
+  return e;
+}
+
+cudaError_t set_smem_once() {
+  static int done[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev >= 0 && dev < 64 && __atomic_load_n(&done[dev], __ATOMIC_ACQUIRE)) return cudaSuccess;
+  e = smem_attrs<attention_tc_kernel<128>, 128>();
+  if (e == cudaSuccess) e = smem_attrs<attention_tc_kernel<64>, 64>();
+  if (e == cudaSuccess && dev >= 0 && dev < 64) __atomic_store_n(&done[dev], 1, __ATOMIC_RELEASE);
+  return e;
+}
+
+static_assert(smem_bytes<128>() <= 232448, "attention kernel shared memory above the opt-in limit");
+
+}  // namespace
+
+size_t attention_tc_workspace(int B, int H, int Mq) {
+  return make_plan(B, H, Mq, 1, 1).acc_bytes;
+}
+
+bool attention_tc_layout_ok(const AttnArgs& a) {
+  if (a.d != 64 && a.d != 128) return false;
+  const void* ptrs[4] = {a.q, a.k, a.v, a.o};
+  for (const void* ptr : ptrs)
+    if (reinterpret_cast<uintptr_t>(ptr) & 15u) return false;
+  for (int i = 0; i < 4; ++i)
+    if (!strides_ok(a.B, a.H, a.str[i][0], a.str[i][1], a.str[i][2])) return false;
+  return encode_fn() != nullptr;
+}
+
+cudaError_t launch_attention_tc(const AttnArgs& a, int num_sms, cudaStream_t s) {
+  const Plan pl = make_plan(a.B, a.H, a.Mq, a.Nk, num_sms);
+  CUtensorMap mq, mk, mv, mo;
+  if (!make_map(&mq, a.q, a.B, a.H, a.Mq, a.d, a.str[0][0], a.str[0][1], a.str[0][2]) ||
+      !make_map(&mk, a.k, a.B, a.H, a.Nk, a.d, a.str[1][0], a.str[1][1], a.str[1][2]) ||
+      !make_map(&mv, a.v, a.B, a.H, a.Nk, a.d, a.str[2][0], a.str[2][1], a.str[2][2]) ||
+      !make_map(&mo, a.o, a.B, a.H, a.Mq, a.d, a.str[3][0], a.str[3][1], a.str[3][2]))
+    return cudaErrorInvalidValue;
+  AttnParams p{};
+  p.B = a.B; p.H = a.H; p.Mq = a.Mq; p.Nk = a.Nk; p.L = a.L;
+  p.n_qp = pl.n_qp; p.n_kt = pl.n_kt; p.n_units = pl.n_units;
+  p.c_log2 = a.scale * 1.4426950408889634f;
+  p.weight = a.weight;
+  p.accumulate = a.accumulate;
+  p.A = a.A;
+  p.lse = a.lse;
+  p.acc = static_cast<unsigned long long*>(a.ws);
+  p.rows_pad = pl.n_qp * kUnitRows;
+  p.status = a.status;
+  cudaError_t e = set_smem_once();
+  if (e != cudaSuccess) return e;
+  if (a.d == 128)
+    e = launch_pdl(attention_tc_kernel<128>, dim3(pl.grid), dim3(kThreads), smem_bytes<128>(), s,
+                   mq, mk, mv, mo, p);
+  else
+    e = launch_pdl(attention_tc_kernel<64>, dim3(pl.grid), dim3(kThreads), smem_bytes<64>(), s,
+                   mq, mk, mv, mo, p);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+}  // namespace avits

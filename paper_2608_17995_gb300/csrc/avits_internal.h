@@ -70,6 +70,27 @@ cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s,
 // CUDA-core path (fp32 or bf16, any d <= 256): one warp per query row.
 cudaError_t launch_spatial_simt(const SpatialArgs& a, cudaStream_t s);
 
+// ---- joint-attention forward (Eq. 4-5) with the spatial score (Eq. 3) -------
+struct AttnArgs {
+  const void* q;     // [B,H,Mq,d] bf16
+  const void* k;     // [B,H,Nk,d] bf16, the L text keys first
+  const void* v;     // [B,H,Nk,d] bf16
+  void* o;           // [B,H,Mq,d] bf16
+  int B, H, Mq, Nk, L, d;
+  int64_t str[4][3];   // element strides (batch, head, row) of q, k, v, o
+  float scale, weight;
+  int accumulate;
+  float* A;          // [B,Mq] or NULL
+  float* lse;        // [B,H,Mq,2] or NULL
+  void* ws;          // head-sum words (A != NULL), zero between calls
+  unsigned int* status;
+};
+// Layout the tensor-core forward takes: d in {64,128}, 16-byte aligned bases
+// and strides.
+bool attention_tc_layout_ok(const AttnArgs& a);
+size_t attention_tc_workspace(int B, int H, int Mq);
+cudaError_t launch_attention_tc(const AttnArgs& a, int num_sms, cudaStream_t s);
+
 // ---- temporal ---------------------------------------------------------------
 // Failure-detection test hook (selftest.cu): bounded waits that cannot complete.
 cudaError_t launch_wait_selftest(unsigned long long limit_ns, long long* result,

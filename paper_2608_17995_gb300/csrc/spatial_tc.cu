@@ -70,9 +70,12 @@
 
 #include "avits_common.cuh"
 #include "avits_internal.h"
+#include "tc_common.cuh"
 
 namespace avits {
 namespace {
+
+using namespace tc;
 
 constexpr int kBM = 128;       // query rows per tile (= TMEM lanes)
 constexpr int kBN = 128;       // keys per tile
@@ -86,6 +89,11 @@ constexpr uint32_t kIdesc = (1u << 4)                       // D: fp32
                             | (1u << 7) | (1u << 10)        // A, B: bf16
                             | ((uint32_t)(kBN >> 3) << 17)  // N
                             | ((uint32_t)(kBM >> 4) << 24); // M
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint32_t a_lo, uint32_t b_lo,
+                                         uint32_t hi, uint32_t acc) {
+  mma_ss(d_tmem, a_lo, b_lo, hi, kIdesc, acc);
+}
 
 template <int D>
 struct Cfg {
@@ -130,115 +138,6 @@ struct TcParams {
   const uint8_t* tmask;   // [B,Nk] text-key mask, or NULL (text keys = the first L)
   const float* lse_all;   // [B,H,M] caller's logsumexp over all keys (natural log), or NULL
 };
-
-// ------------------------------------------------------------------ PTX ----
-__device__ __forceinline__ void tma_load_4d(void* dst, const CUtensorMap* map, int c0, int c1,
-                                            int c2, int c3, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3),
-      "r"(smem_u32(bar))
-      : "memory");
-}
-
-// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row
-// core-matrix groups 1024 B apart.
-__device__ __forceinline__ uint64_t sw128_desc(const void* p) {
-  const uint32_t a = smem_u32(p);
-  return (uint64_t)((a >> 4) & 0x3FFFu) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
-         ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
-}
-
-// The same descriptor as two 32-bit words: the low word holds the start
-// address (bits 0-13, in 16-byte units) and the leading-byte offset, the high
-// word the stride, version and swizzle fields, which are equal for every tile.
-// A K-step moves the start address only (no carry: shared memory < 256 KB), so
-// the issuer adds constants to the low word instead of rebuilding descriptors.
-__device__ __forceinline__ uint32_t sw128_desc_lo(const void* p) {
-  return (uint32_t)sw128_desc(p);
-}
-__device__ __forceinline__ uint32_t sw128_desc_hi() {
-  return (uint32_t)(((uint64_t)(1024 >> 4) << 32 | ((uint64_t)1 << 46) | ((uint64_t)2 << 61)) >> 32);
-}
-
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint32_t a_lo, uint32_t b_lo,
-                                         uint32_t hi, uint32_t acc) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t.reg .b64 ad, bd;\n\t"
-      "setp.ne.b32 p, %5, 0;\n\t"
-      "mov.b64 ad, {%1, %3};\n\tmov.b64 bd, {%2, %3};\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %4, p;\n\t}" ::"r"(d_tmem),
-      "r"(a_lo), "r"(b_lo), "r"(hi), "r"(kIdesc), "r"(acc));
-}
-
-__device__ __forceinline__ void mma_commit(uint64_t* bar) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-          smem_u32(bar))
-      : "memory");
-}
-
-__device__ __forceinline__ void tc_fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-
-#define AVITS_R8(b) "=r"(r[b]), "=r"(r[b + 1]), "=r"(r[b + 2]), "=r"(r[b + 3]), \
-                    "=r"(r[b + 4]), "=r"(r[b + 5]), "=r"(r[b + 6]), "=r"(r[b + 7])
-#define AVITS_W8(b) "+r"(r[b]), "+r"(r[b + 1]), "+r"(r[b + 2]), "+r"(r[b + 3]), \
-                    "+r"(r[b + 4]), "+r"(r[b + 5]), "+r"(r[b + 6]), "+r"(r[b + 7])
-
-// 16 consecutive fp32 columns of this thread's TMEM lane.
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
-      "%11, %12, %13, %14, %15}, [%16];"
-      : AVITS_R8(0), AVITS_R8(8)
-      : "r"(taddr));
-}
-
-// Completes the thread's outstanding tcgen05.ld; the registers are tied to
-// the wait so that no use can be scheduled before it.
-__device__ __forceinline__ void tmem_wait(uint32_t (&r)[16]) {
-  asm volatile("tcgen05.wait::ld.sync.aligned;" : AVITS_W8(0), AVITS_W8(8) : : "memory");
-}
-
-__device__ __forceinline__ float ex2(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
-__device__ __forceinline__ float max3(float a, float b, float c) {
-  float d;
-  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
-  return d;
-}
-
-// (a0, a1) * b + c on both lanes of a packed pair.
-__device__ __forceinline__ void ffma2(float a0, float a1, float b, float c, float& d0, float& d1) {
-  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
-      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %4};\n\tmov.b64 rc, {%5, %5};\n\t"
-      "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
-      : "=f"(d0), "=f"(d1)
-      : "f"(a0), "f"(a1), "f"(b), "f"(c));
-}
-
-// (s0, s1) += (e0, e1) on a packed pair.
-__device__ __forceinline__ void fadd2(float& s0, float& s1, float e0, float e1) {
-  asm("{\n\t.reg .b64 ra, rb;\n\t"
-      "mov.b64 ra, {%0, %1};\n\tmov.b64 rb, {%2, %3};\n\t"
-      "add.rn.f32x2 ra, ra, rb;\n\tmov.b64 {%0, %1}, ra;\n\t}"
-      : "+f"(s0), "+f"(s1)
-      : "f"(e0), "f"(e1));
-}
-
-__device__ __forceinline__ void bar_sync(int id, int count) {
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
-}
 
 // Running row statistics in the log2 domain: x = c_log2 * (q.k); the sums
 // are of 2^(x - m).
@@ -381,29 +280,10 @@ __device__ __forceinline__ bool piece_wait(const unsigned long long* w, unsigned
   return false;
 }
 
-// Fixed-point head sum (Eq. 3): word = heads << 56 | NaN masses << 48 | sum of
-// round(mass * 2^40).  H <= 255, so neither count overflows its byte and the
-// sum stays below 2^48.
-
+// Eq. 3's head sum of this row (fixed point, order independent).
 __device__ __forceinline__ void head_sum_add(const TcParams& p, int b, int row, float mass) {
-  unsigned long long inc = 1ull << 56;
-  if (mass != mass)
-    inc |= 1ull << 48;
-  else
-    inc += __float2ull_rn(fminf(fmaxf(mass, 0.f), 1.f) * 0x1p40f);
-  unsigned long long* w = p.acc + (long long)b * p.rows_pad + row;
-  const unsigned long long v = atomicAdd(w, inc) + inc;
-  if ((int)(v >> 56) != p.H) return;
-  *w = 0ull;   // every head is in: clear the word for the next call
-  float a;
-  if ((v >> 48) & 0xFFull) {
-    a = __int_as_float(0x7fc00000);
-  } else {
-    const double mean = (double)(v & ((1ull << 48) - 1ull)) * 0x1p-40 / (double)p.H;
-    a = (float)((double)p.weight * mean);
-  }
-  float* ap = p.A + (long long)b * p.M + row;
-  *ap = p.accumulate ? *ap + a : a;
+  tc::head_sum_add(p.acc + (long long)b * p.rows_pad + row, p.H, mass, p.weight, p.accumulate,
+                   p.A + (long long)b * p.M + row);
 }
 
 // Kinds of the 64 keys a softmax warp reduces per item.
@@ -493,7 +373,7 @@ __device__ __forceinline__ void softmax_item(uint32_t tb, int c0, int Nk, int L,
   tmem_ld16(tb + 48, rb);
   chunk(ra, 2);
   tmem_wait(rb);
-  tc_fence_before();
+  fence_before();
   __syncwarp();
   if (lane == 0) mbar_arrive(s_empty);
   chunk(rb, 3);
@@ -642,9 +522,9 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
                  "r"(kTmemCols));
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
-  tc_fence_before();
+  fence_before();
   __syncthreads();
-  tc_fence_after();
+  fence_after();
   const uint32_t tmem = bars->tmem_base;
   volatile int* abort_flag = &bars->abort;
   // the next kernel may be scheduled now (it waits for this grid to finish
@@ -752,7 +632,7 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
           }
           ok = mbar_wait_bounded(&bars->s_empty[t][sb], sph ^ 1u, abort_flag, p.status);
           if (!ok) break;
-          tc_fence_after();
+          fence_after();
           const uint32_t d_tmem = d_base + (uint32_t)(sb * kBN);
           const uint32_t b_lo = b_lo0 + (uint32_t)((stage * C::kTileBytes) >> 4);
 #pragma unroll
@@ -800,7 +680,7 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
         bool ok = (*abort_flag == 0) && mbar_wait_bounded(&bars->s_full[t][sb], sph, abort_flag, p.status);
         ok = __all_sync(0xffffffffu, ok);   // tcgen05.ld below is warp-collective
         if (ok) {
-          tc_fence_after();
+          fence_after();
           const uint32_t tb = tlane + (uint32_t)(sb * kBN);
           const int c0 = (seg.kt0 + j) * kBN + half * 64;   // first key of this half
           uint64_t* empty = &bars->s_empty[t][sb];
@@ -851,54 +731,13 @@ spatial_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant
     }
   }
 
-  tc_fence_before();
+  fence_before();
   __syncthreads();
   if (warp == 1) {
-    tc_fence_after();
+    fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                  "r"(kTmemCols));
   }
-}
-
-// ------------------------------------------------------------------ host ---
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
-                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
-                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
-                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn encode_fn() {
-  static EncodeTiledFn fn = nullptr;
-  static bool tried = false;
-  if (!tried) {
-    tried = true;
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiledFn>(p);
-  }
-  return fn;
-}
-
-// Element strides of a [B,H,rows,d] view -> byte strides for the tensor map;
-// a dimension of extent 1 gets a packed stride (its stride is never used).
-bool make_map(CUtensorMap* map, const void* base, int B, int H, int rows, int d, int64_t sb,
-              int64_t sh, int64_t sn) {
-  EncodeTiledFn fn = encode_fn();
-  if (!fn) return false;
-  const int64_t e = 2;
-  int64_t s_n = sn * e;
-  int64_t s_h = (H > 1) ? sh * e : s_n * rows;
-  int64_t s_b = (B > 1) ? sb * e : s_h * H;
-  cuuint64_t dims[4] = {(cuuint64_t)d, (cuuint64_t)rows, (cuuint64_t)H, (cuuint64_t)B};
-  cuuint64_t strides[3] = {(cuuint64_t)s_n, (cuuint64_t)s_h, (cuuint64_t)s_b};
-  cuuint32_t box[4] = {64, 128, 1, 1};
-  cuuint32_t estr[4] = {1, 1, 1, 1};
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides,
-                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  return r == CUDA_SUCCESS;
 }
 
 struct Plan {
@@ -925,13 +764,6 @@ Plan make_plan(int B, int H, int M, int Nk, int num_sms) {
   pl.part_bytes = align256(2 * sizeof(unsigned long long) * (size_t)pl.n_units * pl.max_parts * kUnitRows);
   pl.bytes = pl.acc_bytes + pl.part_bytes;
   return pl;
-}
-
-bool strides_ok(int B, int H, int64_t sb, int64_t sh, int64_t sn) {
-  if (sn % 8 != 0 || sn <= 0) return false;
-  if (H > 1 && (sh % 8 != 0 || sh <= 0)) return false;
-  if (B > 1 && (sb % 8 != 0 || sb <= 0)) return false;
-  return true;
 }
 
 // All-shared carveout and the dynamic shared-memory opt-in of one instance.

@@ -30,6 +30,11 @@ Value recipe (documented draw order, numpy PCG64 ``default_rng(seed)``):
   6. Editing config: R reference keys on the doubled grid,
      K_ref(Y,X) = 0.6 K_img(Y//2, X//2) + 0.8 N(0, var(K_img)), placed after
      the image keys.
+  7. Joint-attention forward (make_joint_attention): one query per key of
+     the joint sequence, Q = [Q_txt; Q_img; Q_ref]; Q_img is step 1-3's,
+     Q_txt and Q_ref ~ N(0, var(K)) (the keys' scale after step 3), and the
+     values V ~ N(0,1) [B,H,Nk,d], drawn from default_rng(seed + 7) in the
+     order Q_txt, Q_ref, V per batch element.
 bf16 tensors are float values rounded to nearest-even bf16 and kept as their
 uint16 bit patterns (numpy has no bfloat16).
 """
@@ -42,7 +47,7 @@ from typing import Dict, List, Optional
 import numpy as np
 
 __all__ = [
-    "Transition", "CONFIGS", "make_transition", "make_batched_stage2",
+    "Transition", "CONFIGS", "make_transition", "make_batched_stage2", "make_joint_attention",
     "to_bf16_bits", "bf16_bits_to_f32", "smooth_field",
 ]
 
@@ -223,6 +228,26 @@ def make_transition(name: str, seed: Optional[int] = None, **overrides) -> Trans
         q_img=_finish(np.stack(qs), dt), k_all=_finish(np.stack(ks), dt),
         h_t=_finish(np.stack(hts), dt), h_prev=_finish(np.stack(hps), dt),
         latent=_finish(np.stack(lats), dt), frame_h=gh, frame_w=gw)
+
+
+def make_joint_attention(tr: "Transition", seed: Optional[int] = None):
+    """Step 7 of the recipe: (q_all [B,H,Nk,d], v_all [B,H,Nk,d]) of the joint
+    sequence of transition ``tr``, rows ordered as its keys (text, image,
+    reference).  Same dtype convention as ``tr``."""
+    s = (CONFIGS[tr.name]["seed"] if seed is None else seed) + 7
+    B, H, L, M, R, d = tr.B, tr.H, tr.L, tr.M, tr.R, tr.d
+    k = bf16_bits_to_f32(tr.k_all) if tr.dtype == "bf16" else tr.k_all
+    q_img = bf16_bits_to_f32(tr.q_img) if tr.dtype == "bf16" else tr.q_img
+    qs, vs = [], []
+    for b in range(B):
+        rng = np.random.default_rng(s + 1000 * b)
+        sd = float(np.std(k[b].astype(np.float64)))
+        q_txt = rng.standard_normal((H, L, d)) * sd
+        q_ref = rng.standard_normal((H, R, d)) * sd
+        v = rng.standard_normal((H, L + M + R, d))
+        qs.append(np.concatenate([q_txt, q_img[b].astype(np.float64), q_ref], axis=1))
+        vs.append(v)
+    return _finish(np.stack(qs), tr.dtype), _finish(np.stack(vs), tr.dtype)
 
 
 def make_batched_stage2(pos: np.ndarray, span: np.ndarray, frame: int, seed: int = 100,

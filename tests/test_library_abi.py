@@ -169,6 +169,40 @@ def test_host_validation_of_the_lse_entry(lib):
     assert f(*args(P, 0, 32, 0.125)) == 2
 
 
+def test_host_validation_of_the_attention_forward(lib):
+    """avits_attention_forward rejects bad arguments on the host: sizes, L,
+    the scale, short row strides and a missing or short workspace when A is
+    wanted (INVALID_ARG); fp32 inputs and H > 255 with A (UNSUPPORTED)."""
+    P = ctypes.c_void_p(256)
+    INVALID, UNSUPPORTED = 1, 2
+    f = lib.avits_attention_forward
+    ws = lib.avits_attention_forward_workspace(1, 2, 300)
+    assert ws == 8 * 512
+    assert lib.avits_attention_forward_workspace(0, 2, 300) == 0
+
+    def call(**kw):
+        a = dict(q=P, k=P, v=P, dt=1, B=1, H=2, Mq=300, Nk=333, L=77, d=128, qs=None, ks=None,
+                 vs=None, os=None, scale=0.088, o=P, lse=None, w=1.0, acc=0, A=P, ws=P, wsb=ws)
+        a.update(kw)
+        return f(a["q"], a["k"], a["v"], a["dt"], a["B"], a["H"], a["Mq"], a["Nk"], a["L"],
+                 a["d"], a["qs"], a["ks"], a["vs"], a["os"], a["scale"], a["o"], a["lse"], a["w"],
+                 a["acc"], a["A"], a["ws"], a["wsb"], None)
+
+    assert call(o=None) == INVALID
+    assert call(Mq=0) == INVALID
+    assert call(L=334) == INVALID
+    assert call(L=-1) == INVALID
+    assert call(scale=0.0) == INVALID
+    assert call(scale=float("nan")) == INVALID
+    short = (ctypes.c_int64 * 3)(0, 0, 64)      # row stride < d
+    assert call(qs=short) == INVALID
+    assert call(ws=None) == INVALID
+    assert call(wsb=ws - 8) == INVALID
+    assert call(ws=ctypes.c_void_p(260)) == INVALID      # not 8-byte aligned
+    assert call(dt=0) == UNSUPPORTED
+    assert call(H=256, wsb=1 << 20) == UNSUPPORTED
+
+
 def test_nvtx_ranges_compile(tmp_path):
     """With AVITS_NVTX the entry points open NVTX ranges (header-only NVTX v3,
     so nothing to link): the entry-point sources compile with it."""
