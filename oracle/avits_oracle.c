@@ -387,14 +387,103 @@ static float bil_combine(float p00, float p01, float p10, float p11, float wy0, 
 }
 
 /* ---------------------------------------------------------------------------
+ * Multi-level bilinear resampling (the reading of "orthogonal upsampling" for
+ * frames that hold tokens of several spans, Sec. 3.2 Stages 2-3).
+ *
+ * A frame of fh x fw cells is tiled by tokens of span s (a power of two, the
+ * token at a multiple of s); its pixel image E (2fh x 2fw) repeats each of a
+ * token's 2x2 pixels over the s x s full pixels it stands for.  The pyramid:
+ * P_0 = E and P_l = the 2x2 average pool of P_(l-1), ((a + b) + (c + d)) *
+ * 0.25 over (2R,2Q), (2R,2Q+1), (2R+1,2Q), (2R+1,2Q+1), except that a level-l
+ * pixel lying inside one token pixel (the token's span >= 2^l) is that pixel
+ * itself.  A selected token of span 2^l is upsampled by the half-pixel-
+ * centred 2x bilinear resize of P_l (Stage 2); the merge refines every token
+ * coarser than level l from level l + 1 the same way, coarsest level first
+ * (Stage 3).  With spans 1 and 2 only this is the single-level rule: P_0 is
+ * the dense latent image, P_1 the rebuilt half-resolution image.
+ * ------------------------------------------------------------------------- */
+typedef struct {
+  const void* mixed;      /* token values of one element, [N, T] */
+  int dtype, T;
+  const int32_t* pos;     /* [N, 2] */
+  const int32_t* span;    /* [N] */
+  const int32_t* owner;   /* [fh * fw] cell -> covering token */
+  int fh, fw;
+} frame_t;
+
+static int is_pow2(int s) { return s > 0 && (s & (s - 1)) == 0; }
+static int log2i(int s) { int l = 0; while ((1 << l) < s) ++l; return l; }
+
+/* owner map of one element's tokens; OR_COVERAGE unless they tile the frame
+ * exactly with power-of-two spans at multiples of their span */
+static int frame_owner(const int32_t* pos, const int32_t* span, int N, int fh, int fw,
+                       int32_t* owner, int32_t* count) {
+  int rc = OR_OK;
+  for (int64_t c = 0; c < (int64_t)fh * fw; ++c) { owner[c] = -1; count[c] = 0; }
+  for (int t = 0; t < N; ++t) {
+    const int y = pos[t * 2], x = pos[t * 2 + 1], s = span[t];
+    if (!is_pow2(s) || y % s || x % s) { rc = OR_COVERAGE; continue; }
+    for (int u = 0; u < s; ++u)
+      for (int v = 0; v < s; ++v) {
+        const int Y = y + u, X = x + v;
+        if (Y < 0 || Y >= fh || X < 0 || X >= fw) { rc = OR_COVERAGE; continue; }
+        count[(int64_t)Y * fw + X]++;
+        owner[(int64_t)Y * fw + X] = t;
+      }
+  }
+  for (int64_t c = 0; c < (int64_t)fh * fw; ++c)
+    if (count[c] != 1) rc = OR_COVERAGE;
+  return rc;
+}
+
+/* P_l(R, Q), channel ch */
+static float pyr_pixel(const frame_t* f, int ch, int l, int R, int Q) {
+  const int Y = R << l, X = Q << l;   /* the block's first full pixel */
+  const int t = f->owner[(int64_t)(Y >> 1) * f->fw + (X >> 1)];
+  const int s = f->span[t];
+  if (s >= (1 << l)) {
+    const int ty = (Y - 2 * f->pos[t * 2]) / s, tx = (X - 2 * f->pos[t * 2 + 1]) / s;
+    return get_f32(f->mixed, f->dtype, (int64_t)t * f->T + ch * 4 + ty * 2 + tx);
+  }
+  volatile float a = pyr_pixel(f, ch, l - 1, 2 * R, 2 * Q);
+  volatile float b = pyr_pixel(f, ch, l - 1, 2 * R, 2 * Q + 1);
+  volatile float c = pyr_pixel(f, ch, l - 1, 2 * R + 1, 2 * Q);
+  volatile float d = pyr_pixel(f, ch, l - 1, 2 * R + 1, 2 * Q + 1);
+  volatile float top = a + b;
+  volatile float bot = c + d;
+  volatile float sum = top + bot;
+  return sum * 0.25f;
+}
+
+/* Stage 3 value of level-l pixel (R, Q): U_L = P_L; below it, a pixel of a
+ * token coarser than 2^l is the 2x bilinear resize of U_(l+1), any other the
+ * frame's own P_l */
+static float cascade_pixel(const frame_t* f, int ch, int l, int L, int R, int Q) {
+  if (l >= L) return pyr_pixel(f, ch, l, R, Q);
+  const int Y = R << l, X = Q << l;
+  const int s = f->span[f->owner[(int64_t)(Y >> 1) * f->fw + (X >> 1)]];
+  if (s <= (1 << l)) return pyr_pixel(f, ch, l, R, Q);
+  const int nh = (2 * f->fh) >> (l + 1), nw = (2 * f->fw) >> (l + 1);
+  int r0, r1, c0, c1;
+  float wy0, wy1, wx0, wx1;
+  bil_axis(R, nh, &r0, &r1, &wy0, &wy1);
+  bil_axis(Q, nw, &c0, &c1, &wx0, &wx1);
+  return bil_combine(cascade_pixel(f, ch, l + 1, L, r0, c0), cascade_pixel(f, ch, l + 1, L, r0, c1),
+                     cascade_pixel(f, ch, l + 1, L, r1, c0), cascade_pixel(f, ch, l + 1, L, r1, c1),
+                     wy0, wy1, wx0, wx1);
+}
+
+/* ---------------------------------------------------------------------------
  * Selective upsampling, Sec. 3.2 Stage 2, p = 2, tokens of C*4 values in
  * (channel, patch row, patch col) order.  Tokens are visited in index order;
  * a selected token at (y,x) with span s becomes 4 children (a,b) at
  * (2y + a*s, 2x + b*s) with span s, child (a,b) being the 2x upsample of the
  * parent's pixel (a,b); a deferred token is copied to (2y, 2x) with span 2s.
- * Nearest: each child pixel equals the parent pixel.  Bilinear (dense single-
- * level grid only): the child pixels are the half-pixel-centred 2x bilinear
- * resize of the dense low-resolution latent image.
+ * Nearest: each child pixel equals the parent pixel.  Bilinear: the children
+ * of a selected token of span 2^l are its pixels in the half-pixel-centred 2x
+ * bilinear resize of level l of the input frame's pyramid (see above; for a
+ * dense grid, level 0 is the latent image itself).  A mixed input (pos_in)
+ * must tile the gh x gw frame; bilinear then also needs gh, gw even.
  * Returns the number of emitted tokens in *n_out.
  * ------------------------------------------------------------------------- */
 int avits_oracle_selective_upsample(const void* latent, int dtype, int B, int M, int gh, int gw,
@@ -404,17 +493,41 @@ int avits_oracle_selective_upsample(const void* latent, int dtype, int B, int M,
                                     int* n_out) {
   if (B <= 0 || M <= 0 || C <= 0 || gh <= 0 || gw <= 0) return OR_BAD_ARG;
   if (!pos_in && M != gh * gw) return OR_BAD_ARG;
-  if (mode == 1 && pos_in) return OR_BAD_ARG;
+  if (mode == 1 && pos_in && ((gh & 1) || (gw & 1))) return OR_BAD_ARG;
   const int T = C * 4;
   int k = 0;
   for (int i = 0; i < M; ++i) k += mask[i] ? 1 : 0;
   const int64_t NO = (int64_t)M + 3 * (int64_t)k;
-  const int IH = 2 * gh, IW = 2 * gw;   /* low-res pixel image (bilinear) */
-  for (int b = 0; b < B; ++b) {
+  /* bilinear: the input frame (its owner map; a dense grid is the frame of
+   * span-1 tokens in raster order) */
+  int32_t *owner = NULL, *cnt = NULL, *dpos = NULL, *dspan = NULL;
+  if (mode == 1) {
+    owner = (int32_t*)malloc(sizeof(int32_t) * (size_t)gh * gw);
+    cnt = (int32_t*)malloc(sizeof(int32_t) * (size_t)gh * gw);
+    if (!pos_in) {
+      dpos = (int32_t*)malloc(sizeof(int32_t) * 2 * (size_t)M);
+      dspan = (int32_t*)malloc(sizeof(int32_t) * (size_t)M);
+      for (int i = 0; i < M; ++i) { dpos[2 * i] = i / gw; dpos[2 * i + 1] = i % gw; dspan[i] = 1; }
+    }
+  }
+  int rc = OR_OK;
+  for (int b = 0; b < B && rc == OR_OK; ++b) {
     int kb = 0;
     for (int i = 0; i < M; ++i) kb += mask[(int64_t)b * M + i] ? 1 : 0;
-    if (kb != k) return OR_BAD_ARG;      /* one k per call */
+    if (kb != k) { rc = OR_BAD_ARG; break; }      /* one k per call */
     const int64_t lbase = (int64_t)b * M * T;
+    frame_t fr;
+    if (mode == 1) {
+      fr.mixed = (const char*)latent + lbase * (dtype == 0 ? 4 : 2);
+      fr.dtype = dtype;
+      fr.T = T;
+      fr.pos = pos_in ? pos_in + (int64_t)b * M * 2 : dpos;
+      fr.span = pos_in ? span_in + (int64_t)b * M : dspan;
+      fr.owner = owner;
+      fr.fh = gh;
+      fr.fw = gw;
+      if (frame_owner(fr.pos, fr.span, M, gh, gw, owner, cnt) != OR_OK) { rc = OR_BAD_ARG; break; }
+    }
     int64_t o = 0;
     for (int i = 0; i < M; ++i) {
       int y, x, s;
@@ -434,16 +547,17 @@ int avits_oracle_selective_upsample(const void* latent, int dtype, int B, int M,
                   if (mode == 0) {
                     v = get_f32(latent, dtype, lbase + (int64_t)i * T + c * 4 + a * 2 + bb);
                   } else {
-                    /* upsampled pixel (4y+2a+ph, 4x+2b+pw) of the 4gh x 4gw image */
+                    /* the parent covers level-l pixels (2y/s + {0,1}, 2x/s + {0,1});
+                     * child (a,b) pixel (ph,pw) is pixel (2(2y/s) + 2a + ph, ...) of
+                     * the 2x resize of P_l ((2gh >> l) x (2gw >> l) pixels) */
+                    const int l = log2i(s);
                     int r0, r1, c0, c1;
                     float wy0, wy1, wx0, wx1;
-                    bil_axis(4 * y + 2 * a + ph, IH, &r0, &r1, &wy0, &wy1);
-                    bil_axis(4 * x + 2 * bb + pw, IW, &c0, &c1, &wx0, &wx1);
-#define PIX(R, Q) get_f32(latent, dtype, lbase + (int64_t)(((R) >> 1) * gw + ((Q) >> 1)) * T + \
-                                               c * 4 + ((R)&1) * 2 + ((Q)&1))
-                    v = bil_combine(PIX(r0, c0), PIX(r0, c1), PIX(r1, c0), PIX(r1, c1), wy0, wy1,
-                                    wx0, wx1);
-#undef PIX
+                    bil_axis(2 * ((2 * y) >> l) + 2 * a + ph, (2 * gh) >> l, &r0, &r1, &wy0, &wy1);
+                    bil_axis(2 * ((2 * x) >> l) + 2 * bb + pw, (2 * gw) >> l, &c0, &c1, &wx0, &wx1);
+                    v = bil_combine(pyr_pixel(&fr, c, l, r0, c0), pyr_pixel(&fr, c, l, r0, c1),
+                                    pyr_pixel(&fr, c, l, r1, c0), pyr_pixel(&fr, c, l, r1, c1),
+                                    wy0, wy1, wx0, wx1);
                   }
                   put_elem(out, dtype, ot * T + c * 4 + ph * 2 + pw, v);
                 }
@@ -466,10 +580,14 @@ int avits_oracle_selective_upsample(const void* latent, int dtype, int B, int M,
         ++o;
       }
     }
-    if (o != NO) return OR_BAD_ARG;
+    if (o != NO) { rc = OR_BAD_ARG; break; }
   }
+  free(owner);
+  free(cnt);
+  free(dpos);
+  free(dspan);
   if (n_out) *n_out = (int)NO;
-  return OR_OK;
+  return rc;
 }
 
 /* ---------------------------------------------------------------------------
@@ -478,9 +596,12 @@ int avits_oracle_selective_upsample(const void* latent, int dtype, int B, int M,
  * (cover_count, optional [B,fh*fw], receives the per-cell count; any count
  * != 1 returns OR_COVERAGE).  Output is in raster order of the frame.
  * Nearest: full-res pixel (Y,X) (Y in [2y, 2y+2s)) takes the token pixel
- * ((Y-2y)/s, (X-2x)/s).  Bilinear (spans 1 and 2 only): span-1 tokens are
- * copied; the half-resolution latent image is rebuilt (a span-2 token gives
- * its own pixels, each 2x2 block of span-1 tokens gives the 2x2 average of its
+ * ((Y-2y)/s, (X-2x)/s).  Bilinear (power-of-two spans at multiples of their
+ * span, fh and fw even, 2fh and 2fw multiples of the largest span): span-1
+ * tokens are copied; every other pixel is the coarse-to-fine cascade of the
+ * multi-level resampling above.  With spans 1 and 2 it is: the
+ * half-resolution latent image is rebuilt (a span-2 token gives its own
+ * pixels, each 2x2 block of span-1 tokens gives the 2x2 average of its
  * child's pixels: pooled (a,b) = ((p00 + p01) + (p10 + p11)) * 0.25 of child
  * (a,b)) and span-2 cells take its 2x bilinear resize (weights as above).
  * ------------------------------------------------------------------------- */
@@ -492,7 +613,6 @@ int avits_oracle_merge_final(const void* mixed, int dtype, int B, int N, const i
   const int64_t F = (int64_t)fh * fw;
   int32_t* owner = (int32_t*)malloc(sizeof(int32_t) * (size_t)F);
   int32_t* cnt = (int32_t*)malloc(sizeof(int32_t) * (size_t)F);
-  float* low = NULL;
   int rc = OR_OK;
   for (int b = 0; b < B && rc == OR_OK; ++b) {
     for (int64_t c = 0; c < F; ++c) { owner[c] = -1; cnt[c] = 0; }
@@ -529,64 +649,40 @@ int avits_oracle_merge_final(const void* mixed, int dtype, int B, int N, const i
               }
         }
     } else {
+      /* bilinear: every token coarser than a level is refined from the level
+       * above, coarsest first (see the multi-level resampling above) */
       if ((fh & 1) || (fw & 1)) { rc = OR_BAD_ARG; break; }
-      const int lh = fh / 2, lw = fw / 2, IH = fh, IW = fw;   /* low-res pixel image IH x IW */
-      if (!low) low = (float*)malloc(sizeof(float) * (size_t)C * IH * IW);
-      for (int ly = 0; ly < lh && rc == OR_OK; ++ly)
-        for (int lx = 0; lx < lw; ++lx) {
-          int t = owner[(int64_t)(2 * ly) * fw + 2 * lx];
-          int s = span[(int64_t)b * N + t];
-          if (s == 2) {
-            if (pos[((int64_t)b * N + t) * 2] != 2 * ly || pos[((int64_t)b * N + t) * 2 + 1] != 2 * lx) {
-              rc = OR_BAD_ARG; break;
-            }
-            for (int c = 0; c < C; ++c)
-              for (int a = 0; a < 2; ++a)
-                for (int bb = 0; bb < 2; ++bb)
-                  low[((int64_t)c * IH + 2 * ly + a) * IW + 2 * lx + bb] =
-                      get_f32(mixed, dtype, mb + (int64_t)t * T + c * 4 + a * 2 + bb);
-          } else if (s == 1) {
-            for (int a = 0; a < 2; ++a)
-              for (int bb = 0; bb < 2; ++bb) {
-                int tc = owner[(int64_t)(2 * ly + a) * fw + 2 * lx + bb];
-                if (span[(int64_t)b * N + tc] != 1) { rc = OR_BAD_ARG; break; }
-                for (int c = 0; c < C; ++c) {
-                  const int64_t e = mb + (int64_t)tc * T + c * 4;
-                  volatile float top = get_f32(mixed, dtype, e + 0) + get_f32(mixed, dtype, e + 1);
-                  volatile float bot = get_f32(mixed, dtype, e + 2) + get_f32(mixed, dtype, e + 3);
-                  volatile float sum = top + bot;
-                  low[((int64_t)c * IH + 2 * ly + a) * IW + 2 * lx + bb] = sum * 0.25f;
-                }
-              }
-          } else { rc = OR_BAD_ARG; break; }
+      int smax = 1;
+      for (int t = 0; t < N; ++t) {
+        const int s = span[(int64_t)b * N + t];
+        if (!is_pow2(s) || pos[((int64_t)b * N + t) * 2] % s || pos[((int64_t)b * N + t) * 2 + 1] % s) {
+          rc = OR_BAD_ARG;
+          break;
         }
+        if (s > smax) smax = s;
+      }
       if (rc != OR_OK) break;
+      const int L = log2i(smax);
+      if (((2 * fh) >> L) << L != 2 * fh || ((2 * fw) >> L) << L != 2 * fw) { rc = OR_BAD_ARG; break; }
+      frame_t fr;
+      fr.mixed = (const char*)mixed + mb * (dtype == 0 ? 4 : 2);
+      fr.dtype = dtype;
+      fr.T = T;
+      fr.pos = pos + (int64_t)b * N * 2;
+      fr.span = span + (int64_t)b * N;
+      fr.owner = owner;
+      fr.fh = fh;
+      fr.fw = fw;
       for (int Y = 0; Y < fh; ++Y)
-        for (int X = 0; X < fw; ++X) {
-          int t = owner[(int64_t)Y * fw + X];
-          int s = span[(int64_t)b * N + t];
+        for (int X = 0; X < fw; ++X)
           for (int c = 0; c < C; ++c)
             for (int ph = 0; ph < 2; ++ph)
-              for (int pw = 0; pw < 2; ++pw) {
-                float v;
-                if (s == 1) {
-                  v = get_f32(mixed, dtype, mb + (int64_t)t * T + c * 4 + ph * 2 + pw);
-                } else {
-                  int r0, r1, c0, c1;
-                  float wy0, wy1, wx0, wx1;
-                  bil_axis(2 * Y + ph, IH, &r0, &r1, &wy0, &wy1);
-                  bil_axis(2 * X + pw, IW, &c0, &c1, &wx0, &wx1);
-                  const float* L0 = low + (int64_t)c * IH * IW;
-                  v = bil_combine(L0[r0 * IW + c0], L0[r0 * IW + c1], L0[r1 * IW + c0],
-                                  L0[r1 * IW + c1], wy0, wy1, wx0, wx1);
-                }
-                put_elem(out, dtype, ob + ((int64_t)Y * fw + X) * T + c * 4 + ph * 2 + pw, v);
-              }
-        }
+              for (int pw = 0; pw < 2; ++pw)
+                put_elem(out, dtype, ob + ((int64_t)Y * fw + X) * T + c * 4 + ph * 2 + pw,
+                         cascade_pixel(&fr, c, 0, L, 2 * Y + ph, 2 * X + pw));
     }
   }
   free(owner);
   free(cnt);
-  free(low);
   return rc;
 }

@@ -571,3 +571,121 @@ def test_bf16_rounding_is_nearest_even(oracle_mod):
     out32 = oracle_mod.selective_upsample(as_f32(latb), gh, gw, mask, mode="bilinear")[0]
     ref = torch.from_numpy(out32).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
     assert np.array_equal(outb, ref)
+
+
+# ------------------------------------- multi-level bilinear (Sec. 3.2, Stages 2-3)
+
+def _bil2x(img):
+    import torch
+    return torch.nn.functional.interpolate(torch.from_numpy(np.ascontiguousarray(img)),
+                                           scale_factor=2, mode="bilinear",
+                                           align_corners=False).numpy()
+
+
+def _mixed_image(out, pos, span, fh, fw):
+    """Pixel image of a mixed sequence (each token pixel over its s x s footprint)."""
+    B, N, T = out.shape
+    C = T // 4
+    img = np.zeros((B, C, 2 * fh, 2 * fw), np.float32)
+    for b in range(B):
+        for t in range(N):
+            y, x = pos[b, t]
+            s = span[b, t]
+            pix = out[b, t].reshape(C, 2, 2)
+            img[b, :, 2 * y:2 * y + 2 * s, 2 * x:2 * x + 2 * s] = np.repeat(np.repeat(pix, s, 1), s, 2)
+    return img
+
+
+@pytest.mark.parametrize("first", ["all", "none"])
+def test_multilevel_bilinear_two_transitions_all_selected(oracle_mod, first):
+    """Two transitions in bilinear mode with every token selected at the
+    second: after an all-selected first transition the children are the 2x
+    bilinear resize of the 2x resize of the latent (torch, twice); after an
+    all-deferred first one (span-2 tokens, whose level-1 image is the latent
+    itself) they are its single 2x resize.  Merging the all-deferred-then-
+    selected sequence (span 2 everywhere) gives the twice-resized latent."""
+    B, g, C = 2, 4, 3
+    lat = _dense_case(21, B, g, g, C)
+    img = tokens_to_image(lat, g, g)
+    m1 = np.full((B, g * g), 1 if first == "all" else 0, np.uint8)
+    o1, p1, s1, _, _ = oracle_mod.selective_upsample(lat, g, g, m1, mode="bilinear")
+    N1 = o1.shape[1]
+    o2, p2, s2, _, _ = oracle_mod.selective_upsample(o1, 2 * g, 2 * g, np.ones((B, N1), np.uint8),
+                                                     mode="bilinear", pos_in=p1, span_in=s1)
+    got = _mixed_image(o2, p2, s2, 4 * g, 4 * g)
+    if first == "all":
+        ref = _bil2x(_bil2x(img))
+        assert np.all(s2 == 1)
+    else:
+        ref = np.repeat(np.repeat(_bil2x(img), 2, 2), 2, 3)   # span-2 children, one pixel per 2x2
+        assert np.all(s2 == 2)
+    np.testing.assert_allclose(got, ref, rtol=0, atol=2e-6)
+    full, cover = oracle_mod.merge_final(o2, p2, s2, 4 * g, 4 * g, mode="bilinear")
+    assert np.all(cover == 1)
+    np.testing.assert_allclose(tokens_to_image(full, 4 * g, 4 * g), _bil2x(_bil2x(img)), rtol=0,
+                               atol=3e-6)
+
+
+def test_multilevel_merge_of_span4_tokens_is_two_resizes(oracle_mod):
+    """Two all-deferred transitions leave span-4 tokens only; the merge's
+    cascade (level 2 = the latent, level 1 its 2x resize, level 0 that one's)
+    equals torch's bilinear 2x applied twice."""
+    B, g, C = 1, 4, 2
+    lat = _dense_case(22, B, g, g, C)
+    o1, p1, s1, _, _ = oracle_mod.selective_upsample(lat, g, g, np.zeros((B, g * g), np.uint8))
+    o2, p2, s2, _, _ = oracle_mod.selective_upsample(o1, 2 * g, 2 * g, np.zeros((B, g * g), np.uint8),
+                                                     pos_in=p1, span_in=s1)
+    assert np.all(s2 == 4)
+    full, _ = oracle_mod.merge_final(o2, p2, s2, 4 * g, 4 * g, mode="bilinear")
+    img = tokens_to_image(lat, g, g)
+    np.testing.assert_allclose(tokens_to_image(full, 4 * g, 4 * g), _bil2x(_bil2x(img)), rtol=0,
+                               atol=3e-6)
+
+
+def test_multilevel_bilinear_constant_and_copies(oracle_mod):
+    """Random selections at both transitions (spans 1, 2 and 4 mixed): a
+    constant latent stays exactly constant through both upsamples and the
+    merge (the weights sum to one and 1.5 * 0.25 etc. are exact), and the
+    merge copies every span-1 token verbatim."""
+    from paper_2608_17995_gb300.workloads import random_scores
+    B, g, C = 2, 8, 2
+    lat = np.full((B, g * g, 4 * C), 1.5, np.float32)
+    _, m1, _ = oracle_mod.topk(random_scores(3, B, g * g)[0], 20)
+    o1, p1, s1, _, _ = oracle_mod.selective_upsample(lat, g, g, m1, mode="bilinear")
+    _, m2, _ = oracle_mod.topk(random_scores(4, B, o1.shape[1])[0], 40)
+    o2, p2, s2, _, _ = oracle_mod.selective_upsample(o1, 2 * g, 2 * g, m2, mode="bilinear",
+                                                     pos_in=p1, span_in=s1)
+    assert set(np.unique(s2)) == {1, 2, 4}
+    assert np.all(o2 == np.float32(1.5))
+    full, _ = oracle_mod.merge_final(o2, p2, s2, 4 * g, 4 * g, mode="bilinear")
+    assert np.all(full == np.float32(1.5))
+    lat = _dense_case(23, B, g, g, C)
+    o1, p1, s1, _, _ = oracle_mod.selective_upsample(lat, g, g, m1, mode="bilinear")
+    o2, p2, s2, _, _ = oracle_mod.selective_upsample(o1, 2 * g, 2 * g, m2, mode="bilinear",
+                                                     pos_in=p1, span_in=s1)
+    full, _ = oracle_mod.merge_final(o2, p2, s2, 4 * g, 4 * g, mode="bilinear")
+    fw = 4 * g
+    for b in range(B):
+        for t in np.nonzero(s2[b] == 1)[0]:
+            y, x = p2[b, t]
+            assert np.array_equal(full[b, y * fw + x], o2[b, t])
+
+
+def test_multilevel_bilinear_rejects_unaligned_or_odd_frames(oracle_mod):
+    """A mixed bilinear input must tile an even frame with aligned power-of-two
+    spans: an odd frame and a span-3 token are refused, and so is a merge
+    with a token moved off its alignment."""
+    lat = _dense_case(24, 1, 2, 2, 1)
+    out, pos, span, _, _ = oracle_mod.selective_upsample(lat, 2, 2, np.zeros((1, 4), np.uint8))
+    with pytest.raises(ValueError):
+        oracle_mod.selective_upsample(out, 3, 4, np.ones((1, 4), np.uint8), mode="bilinear",
+                                      pos_in=pos, span_in=span)
+    bad = span.copy()
+    bad[0, 0] = 3
+    with pytest.raises(ValueError):
+        oracle_mod.selective_upsample(out, 4, 4, np.ones((1, 4), np.uint8), mode="bilinear",
+                                      pos_in=pos, span_in=bad)
+    shifted = pos.copy()
+    shifted[0, 3] = (1, 3)   # a span-2 token off its alignment (and the tiling)
+    with pytest.raises(ValueError):
+        oracle_mod.merge_final(out, shifted, span, 4, 4, mode="bilinear")
