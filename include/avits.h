@@ -351,14 +351,25 @@ avits_status avits_fuse_select_perturbed(const float* A, const float* V, const f
  *              (2y + a*s, 2x + b*s), span s, each child = 2x upsample of
  *              parent pixel (a,b): nearest broadcasts it; bilinear uses the
  *              fixed weights 0.75/0.25 of a half-pixel-centred 2x resize with
- *              edge clamping over the dense input latent.
+ *              edge clamping over the input's pixel image at the token's own
+ *              resolution: the dense latent, or for a mixed input of spans
+ *              1, 2 and 4, level log2(s) of the input frame's pyramid (a
+ *              pixel inside one token pixel is that pixel, any other the
+ *              ((a + b) + (c + d)) / 4 average of the four pixels below it).
  *   deferred : the token unchanged at (2y, 2x), span 2s.
  * Output positions are in the doubled frame (2gh x 2gw), usable directly as
  * 2D RoPE ids.
  *
  * latent : [B,M,C*4] bf16/fp32.  Without pos_in, M = gh*gw (a dense grid).
  * pos_in_opt/span_in_opt : NULL, or [B,M,2] / [B,M] int32 for a mixed input
- *          (a second transition); nearest mode only.
+ *          (a second transition) on a gh x gw frame.  In bilinear mode the
+ *          tokens must tile the frame with spans 1, 2 or 4 at multiples of
+ *          their span, gh and gw even (AVITS_ERR_COVERAGE on the device
+ *          otherwise).
+ * workspace/ws_bytes : bilinear mode with a mixed input only:
+ *          avits_selective_upsample_workspace() bytes, 16-byte aligned, any
+ *          contents (the call rebuilds the frame's cell map there); otherwise
+ *          ignored (may be NULL).
  * sel_mask, tok_offset : from avits_fuse_select.  k = number selected.
  * out_latent : [B,M+3k,C*4] same dtype.  out_pos : [B,M+3k,2] (row, col).
  * out_span : [B,M+3k].  out_src_tok : [B,M+3k] input token index.
@@ -370,7 +381,13 @@ avits_status avits_selective_upsample(const void* latent, avits_dtype dt, int B,
                                       const uint8_t* sel_mask, const int32_t* tok_offset, int k,
                                       avits_upmode mode, void* out_latent, int32_t* out_pos,
                                       int32_t* out_span, int32_t* out_src_tok,
-                                      int8_t* out_src_sub, void* stream);
+                                      int8_t* out_src_sub, void* workspace, size_t ws_bytes,
+                                      void* stream);
+
+/* Workspace bytes of avits_selective_upsample / avits_select_upsample in
+ * bilinear mode (the input frame's cell map, needed with a mixed input only);
+ * 0 for nearest mode or invalid sizes. */
+size_t avits_selective_upsample_workspace(avits_upmode mode, int B, int grid_h, int grid_w);
 
 /* ------------------------------------------------------------------------
  * avits_fuse_select_perturbed followed by avits_selective_upsample, in ONE
@@ -391,7 +408,8 @@ avits_status avits_select_upsample(const float* A, const float* V, const float* 
                                    int C, int p, const int32_t* pos_in_opt,
                                    const int32_t* span_in_opt, avits_upmode mode,
                                    void* out_latent, int32_t* out_pos, int32_t* out_span,
-                                   int32_t* out_src_tok, int8_t* out_src_sub, void* stream);
+                                   int32_t* out_src_tok, int8_t* out_src_sub, void* workspace,
+                                   size_t ws_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
  * Final merge, Sec. 3.2 Stage 3: expand every remaining token to full
@@ -401,10 +419,16 @@ avits_status avits_select_upsample(const float* A, const float* V, const float* 
  * a cell covered twice, a cell left uncovered and a token outside the frame
  * each raise AVITS_ERR_COVERAGE on the device, in both modes.
  *   nearest  : full-res pixel (Y,X) takes token pixel ((Y-2y)/s, (X-2x)/s).
- *   bilinear : only for spans {1,2} (one transition): span-1 tokens are
- *              copied; the low-res grid is rebuilt (span-2 tokens as they are,
- *              each group of 4 span-1 children 2x2 average pooled) and the
- *              span-2 cells take its half-pixel-centred 2x bilinear resize.
+ *   bilinear : spans 1, 2 and 4 at multiples of their span, full_h and
+ *              full_w even: span-1 tokens are copied; every coarser token is
+ *              refined level by level from the frame's pixel pyramid,
+ *              coarsest first: inside a span-4 token, level 1 is the
+ *              half-pixel-centred 2x bilinear resize of level 2; then every
+ *              cell of span 2 or 4 takes the 2x bilinear resize of level 1.
+ *              With spans 1 and 2 only: the low-res grid is rebuilt (span-2
+ *              tokens as they are, each group of 4 span-1 children 2x2
+ *              average pooled) and the span-2 cells take its 2x resize.  Any
+ *              other span raises AVITS_ERR_COVERAGE.
  * mixed : [B,N,C*4].  pos [B,N,2], span [B,N] int32.
  * out_full : [B,full_h*full_w,C*4] same dtype.
  * workspace : avits_merge_final_workspace() bytes (both modes), 16-byte

@@ -95,9 +95,11 @@ def lib():
         "avits_fuse_select": [vp, vp, i32, i32, f32, f32, i32, vp, vp, vp, vp, vp],
         "avits_fuse_select_perturbed": [vp, vp, vp, i32, i32, f32, f32, i32, vp, vp, vp, vp, vp],
         "avits_selective_upsample": [vp, i32, i32, i32, i32, i32, i32, i32, vp, vp, vp, vp, i32,
-                                     i32, vp, vp, vp, vp, vp, vp],
+                                     i32, vp, vp, vp, vp, vp, vp, sz, vp],
+        "avits_selective_upsample_workspace": [i32, i32, i32, i32],
         "avits_select_upsample": [vp, vp, vp, i32, i32, f32, f32, i32, vp, vp, vp, vp, vp, i32,
-                                  i32, i32, i32, i32, vp, vp, i32, vp, vp, vp, vp, vp, vp],
+                                  i32, i32, i32, i32, vp, vp, i32, vp, vp, vp, vp, vp, vp, sz,
+                                  vp],
         "avits_merge_final": [vp, i32, i32, i32, vp, vp, i32, i32, i32, i32, i32, vp, vp, sz, vp],
         "avits_merge_final_workspace": [i32, i32, i32, i32],
         "avits_score_spatial_noalloc": [vp, vp, i32, i32, i32, i32, i32, i32, i32, i64, i64, i64,
@@ -115,7 +117,8 @@ def lib():
         fn.argtypes = args
         fn.restype = ctypes.c_int
     for name in ("avits_score_spatial_workspace", "avits_merge_final_workspace",
-                 "avits_score_spatial_noalloc_limit", "avits_attention_forward_workspace"):
+                 "avits_score_spatial_noalloc_limit", "avits_attention_forward_workspace",
+                 "avits_selective_upsample_workspace"):
         getattr(L, name).restype = ctypes.c_size_t
     for name in ("avits_status_string", "avits_last_error_string", "avits_version",
                  "avits_score_spatial_noalloc_error"):
@@ -407,31 +410,53 @@ def avits_fuse_select(A, V, alpha: float, k: int, sel_idx, tok_offset, S=None, s
     return sel_idx
 
 
+def avits_selective_upsample_workspace(mode: int, B: int, grid_h: int, grid_w: int) -> int:
+    return int(lib().avits_selective_upsample_workspace(int(mode), B, grid_h, grid_w))
+
+
+def _upsample_ws(mode, pos_in, B, grid_h, grid_w, workspace, device):
+    """The cell-map workspace a mixed bilinear upsample needs (else none)."""
+    if mode != BILINEAR or pos_in is None:
+        return None, 0
+    need = avits_selective_upsample_workspace(mode, B, grid_h, grid_w)
+    if workspace is None:
+        workspace = _torch().empty(need, dtype=_torch().uint8, device=device)
+    return workspace, workspace.numel() * workspace.element_size()
+
+
 def avits_select_upsample(A, V, alpha: float, k: int, sel_idx, tok_offset, sel_mask, latent,
                           grid_h: int, grid_w: int, out_latent, out_pos, out_span, out_src_tok,
                           out_src_sub, S=None, perturb=None, mode: int = NEAREST, pos_in=None,
-                          span_in=None, eps_norm: float = 1e-6, stream=None):
+                          span_in=None, eps_norm: float = 1e-6, workspace=None, stream=None):
     """avits_fuse_select(_perturbed) + avits_selective_upsample in one launch;
     the same outputs as the two calls."""
     B, M = A.shape
     T = latent.shape[2]
+    ws, wb = _upsample_ws(mode, pos_in, B, grid_h, grid_w, workspace, latent.device)
     rc = lib().avits_select_upsample(
         _ptr(A), _ptr(V), _ptr(perturb), B, M, float(alpha), float(eps_norm), int(k), _ptr(S),
         _ptr(sel_idx), _ptr(sel_mask), _ptr(tok_offset), _ptr(latent), _dtype_code(latent),
         grid_h, grid_w, T // 4, 2, _ptr(pos_in), _ptr(span_in), int(mode), _ptr(out_latent),
-        _ptr(out_pos), _ptr(out_span), _ptr(out_src_tok), _ptr(out_src_sub), _stream(stream))
+        _ptr(out_pos), _ptr(out_span), _ptr(out_src_tok), _ptr(out_src_sub), _ptr(ws), wb,
+        _stream(stream))
     _check("avits_select_upsample", rc)
     return sel_idx
 
 
 def avits_selective_upsample(latent, grid_h: int, grid_w: int, sel_mask, tok_offset, k: int,
                              out_latent, out_pos, out_span, out_src_tok, out_src_sub,
-                             mode: int = NEAREST, pos_in=None, span_in=None, stream=None):
+                             mode: int = NEAREST, pos_in=None, span_in=None, workspace=None,
+                             stream=None):
+    """Sec. 3.2 Stage 2.  A mixed bilinear input (pos_in given) needs
+    avits_selective_upsample_workspace() bytes of scratch (allocated here when
+    ``workspace`` is None)."""
     B, M, T = latent.shape
+    ws, wb = _upsample_ws(mode, pos_in, B, grid_h, grid_w, workspace, latent.device)
     rc = lib().avits_selective_upsample(
         _ptr(latent), _dtype_code(latent), B, M, grid_h, grid_w, T // 4, 2, _ptr(pos_in),
         _ptr(span_in), _ptr(sel_mask), _ptr(tok_offset), int(k), int(mode), _ptr(out_latent),
-        _ptr(out_pos), _ptr(out_span), _ptr(out_src_tok), _ptr(out_src_sub), _stream(stream))
+        _ptr(out_pos), _ptr(out_span), _ptr(out_src_tok), _ptr(out_src_sub), _ptr(ws), wb,
+        _stream(stream))
     _check("avits_selective_upsample", rc)
     return out_latent
 

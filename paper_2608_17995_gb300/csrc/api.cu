@@ -36,6 +36,15 @@ avits_status cuda_status(cudaError_t e) {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 bool valid_dtype(avits_dtype dt) { return dt == AVITS_F32 || dt == AVITS_BF16; }
 
+// A mixed input in bilinear mode needs the cell map of its frame: an even
+// frame, token indices that fit the map entry, and the workspace.
+bool mixed_bilinear_ok(avits_upmode mode, const int32_t* pos_in, int B, int M, int gh, int gw,
+                       const void* ws, size_t ws_bytes) {
+  if (mode != AVITS_UP_BILINEAR || !pos_in) return true;
+  if ((gh & 1) || (gw & 1) || M > (1 << 28) - 1) return false;
+  return ws && aligned16(ws) && ws_bytes >= merge_workspace_bytes(B, gh, gw);
+}
+
 }  // namespace
 
 // The device address of g_status on the current device, looked up once per
@@ -293,7 +302,8 @@ avits_status avits_selective_upsample(const void* latent, avits_dtype dt, int B,
                                       const uint8_t* sel_mask, const int32_t* tok_offset, int k,
                                       avits_upmode mode, void* out_latent, int32_t* out_pos,
                                       int32_t* out_span, int32_t* out_src_tok,
-                                      int8_t* out_src_sub, void* stream) {
+                                      int8_t* out_src_sub, void* workspace, size_t ws_bytes,
+                                      void* stream) {
   AVITS_RANGE();
   if (!latent || !sel_mask || !tok_offset || !out_latent || !out_pos || !out_span ||
       !out_src_tok || !out_src_sub || !valid_dtype(dt))
@@ -304,12 +314,18 @@ avits_status avits_selective_upsample(const void* latent, avits_dtype dt, int B,
   if ((pos_in_opt == nullptr) != (span_in_opt == nullptr)) return AVITS_ERR_INVALID_ARG;
   if (!pos_in_opt && (int64_t)grid_h * grid_w != M) return AVITS_ERR_INVALID_ARG;
   if (mode != AVITS_UP_NEAREST && mode != AVITS_UP_BILINEAR) return AVITS_ERR_INVALID_ARG;
-  if (mode == AVITS_UP_BILINEAR && pos_in_opt) return AVITS_ERR_UNSUPPORTED;
   if (!aligned16(latent) || !aligned16(out_latent)) return AVITS_ERR_INVALID_ARG;
+  if (!mixed_bilinear_ok(mode, pos_in_opt, B, M, grid_h, grid_w, workspace, ws_bytes))
+    return AVITS_ERR_INVALID_ARG;
   return cuda_status(launch_upsample(latent, dt, B, M, grid_h, grid_w, C, pos_in_opt, span_in_opt,
                                      sel_mask, tok_offset, k, mode, out_latent, out_pos, out_span,
-                                     out_src_tok, out_src_sub,
+                                     out_src_tok, out_src_sub, workspace, status_word(),
                                      static_cast<cudaStream_t>(stream)));
+}
+
+size_t avits_selective_upsample_workspace(avits_upmode mode, int B, int grid_h, int grid_w) {
+  if (mode != AVITS_UP_BILINEAR || B <= 0 || grid_h <= 0 || grid_w <= 0) return 0;
+  return merge_workspace_bytes(B, grid_h, grid_w);
 }
 
 avits_status avits_select_upsample(const float* A, const float* V, const float* perturb, int B,
@@ -319,7 +335,8 @@ avits_status avits_select_upsample(const float* A, const float* V, const float* 
                                    int C, int p, const int32_t* pos_in_opt,
                                    const int32_t* span_in_opt, avits_upmode mode,
                                    void* out_latent, int32_t* out_pos, int32_t* out_span,
-                                   int32_t* out_src_tok, int8_t* out_src_sub, void* stream) {
+                                   int32_t* out_src_tok, int8_t* out_src_sub, void* workspace,
+                                   size_t ws_bytes, void* stream) {
   AVITS_RANGE();
   if (!A || !V || !tok_offset || !sel_mask || (k > 0 && !sel_idx)) return AVITS_ERR_INVALID_ARG;
   if (B <= 0 || M <= 0 || M > kSelectMaxM || k < 0 || k > M) return AVITS_ERR_INVALID_ARG;
@@ -332,12 +349,13 @@ avits_status avits_select_upsample(const float* A, const float* V, const float* 
   if ((pos_in_opt == nullptr) != (span_in_opt == nullptr)) return AVITS_ERR_INVALID_ARG;
   if (!pos_in_opt && (int64_t)grid_h * grid_w != M) return AVITS_ERR_INVALID_ARG;
   if (mode != AVITS_UP_NEAREST && mode != AVITS_UP_BILINEAR) return AVITS_ERR_INVALID_ARG;
-  if (mode == AVITS_UP_BILINEAR && pos_in_opt) return AVITS_ERR_UNSUPPORTED;
   if (!aligned16(latent) || !aligned16(out_latent)) return AVITS_ERR_INVALID_ARG;
+  if (!mixed_bilinear_ok(mode, pos_in_opt, B, M, grid_h, grid_w, workspace, ws_bytes))
+    return AVITS_ERR_INVALID_ARG;
   return cuda_status(launch_select_upsample(
       A, V, perturb, B, M, alpha, eps_norm, k, S_opt, sel_idx, sel_mask, tok_offset,
       status_word(), latent, dt, grid_h, grid_w, C, pos_in_opt, span_in_opt, mode, out_latent,
-      out_pos, out_span, out_src_tok, out_src_sub, static_cast<cudaStream_t>(stream)));
+      out_pos, out_span, out_src_tok, out_src_sub, workspace, static_cast<cudaStream_t>(stream)));
 }
 
 size_t avits_merge_final_workspace(avits_upmode mode, int B, int full_h, int full_w) {
@@ -357,7 +375,8 @@ avits_status avits_merge_final(const void* mixed, avits_dtype dt, int B, int N, 
   if (p != 2) return AVITS_ERR_UNSUPPORTED;
   if (mode != AVITS_UP_NEAREST && mode != AVITS_UP_BILINEAR) return AVITS_ERR_INVALID_ARG;
   if (!aligned16(mixed) || !aligned16(out_full)) return AVITS_ERR_INVALID_ARG;
-  if (mode == AVITS_UP_BILINEAR && ((full_h & 1) || (full_w & 1))) return AVITS_ERR_INVALID_ARG;
+  if (mode == AVITS_UP_BILINEAR && ((full_h & 1) || (full_w & 1) || N > (1 << 28) - 1))
+    return AVITS_ERR_INVALID_ARG;
   if (!workspace || !aligned16(workspace) ||
       ws_bytes < avits_merge_final_workspace(mode, B, full_h, full_w))
     return AVITS_ERR_INVALID_ARG;

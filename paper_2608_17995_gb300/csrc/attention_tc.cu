@@ -81,6 +81,7 @@ struct Bars {
   uint64_t kv_full[kMaxStages], kv_empty[kMaxStages];
   uint64_t s_full[kQTiles], p_full[kQTiles], pv_done[kQTiles];
   uint64_t o_full[kQTiles], o_empty[kQTiles], drain[kQTiles];
+  uint64_t t1_go;   // one phase: tile 0's first P is written
   uint32_t tmem_base;
   int abort;
 };
@@ -316,6 +317,7 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
       mbar_init(&bars->o_empty[t], 4);
       mbar_init(&bars->drain[t], 1);
     }
+    mbar_init(&bars->t1_go, 4);
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&bars->kv_full[s], 1);
       mbar_init(&bars->kv_empty[s], kQTiles);   // one commit per issuer
@@ -415,6 +417,10 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
           ok = mbar_wait_bounded(&bars->kv_full[sk], (uint32_t)((lk / C::kStages) & 1), abort_flag, p.status);
           if (ok && j == 0)
             ok = mbar_wait_bounded(&bars->q_full[t], (uint32_t)(ui & 1), abort_flag, p.status);
+          // tile 1 starts one softmax behind tile 0, so that the two tiles'
+          // S, softmax and PV stages overlap instead of running in lockstep
+          if (ok && t == 1 && gi == 0)
+            ok = mbar_wait_bounded(&bars->t1_go, 0u, abort_flag, p.status);
           // P_t of the previous key tile has been read by its PV product
           if (ok && gi > 0)
             ok = mbar_wait_bounded(&bars->pv_done[t], (uint32_t)((gi - 1) & 1), abort_flag, p.status);
@@ -478,7 +484,10 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
           fence_before();
         }
         __syncwarp();
-        if (ok && lane == 0) mbar_arrive(&bars->p_full[t]);
+        if (ok && lane == 0) {
+          mbar_arrive(&bars->p_full[t]);
+          if (t == 0 && gi == 0) mbar_arrive(&bars->t1_go);
+        }
       }
       // ---- epilogue: O / l -> bf16 -> swizzled staging -> TMA store
       ok = ok && (*abort_flag == 0) &&

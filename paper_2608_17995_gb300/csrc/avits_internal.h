@@ -123,15 +123,19 @@ cudaError_t launch_select_upsample(const float* A, const float* V, const float* 
                                    int gh, int gw, int C, const int32_t* pos_in,
                                    const int32_t* span_in, avits_upmode mode, void* out,
                                    int32_t* out_pos, int32_t* out_span, int32_t* out_src_tok,
-                                   int8_t* out_src_sub, cudaStream_t s);
+                                   int8_t* out_src_sub, void* ws, cudaStream_t s);
+// ws: merge_workspace_bytes(B, gh, gw) bytes, 16-byte aligned, used (for the
+// input frame's cell map) only in bilinear mode with a mixed input.
 cudaError_t launch_upsample(const void* latent, avits_dtype dt, int B, int M, int gh, int gw,
                             int C, const int32_t* pos_in, const int32_t* span_in,
                             const uint8_t* mask, const int32_t* tok_offset, int k,
                             avits_upmode mode, void* out, int32_t* out_pos, int32_t* out_span,
-                            int32_t* out_src_tok, int8_t* out_src_sub, cudaStream_t s);
+                            int32_t* out_src_tok, int8_t* out_src_sub, void* ws,
+                            unsigned int* status, cudaStream_t s);
 
 // ---- final merge (Stage 3) --------------------------------------------------
-// Workspace of either mode: a 16-byte header and one 32-bit word per cell.
+// Workspace of either mode (and of a mixed bilinear upsample): a 16-byte
+// header and one 32-bit word per cell.
 size_t merge_workspace_bytes(int B, int fh, int fw);
 cudaError_t launch_merge(const void* mixed, avits_dtype dt, int B, int N, const int32_t* pos,
                          const int32_t* span, int fh, int fw, int C, avits_upmode mode,

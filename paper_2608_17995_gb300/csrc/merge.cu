@@ -11,16 +11,17 @@
 // the CTA count compares the claimed total with B * fh * fw (fewer = a hole,
 // since no cell was claimed twice), clears the word and advances the tag
 // for the next call.  The map needs no clearing between calls.
-// Bilinear (spans 1 and 2): a cell map is scattered first (atomicExch into a
-// -1-filled workspace, so double cover and holes are detected), then every
-// output (cell, channel) gathers: span-1 cells are copied, span-2 cells take
-// the half-pixel-centred 2x bilinear resize of the rebuilt low-res grid, in
-// which each 2x2 block of span-1 tokens contributes its 2x2 average pools.
+// Bilinear (spans 1, 2 and 4): a cell map is scattered first (atomicExch into
+// a -1-filled workspace, so double cover and holes are detected), then every
+// output (cell, channel) gathers: span-1 cells are copied, coarser cells take
+// the half-pixel-centred 2x bilinear resize of level 1 of the frame's pixel
+// pyramid (frame_map.cuh), refined first from level 2 inside span-4 tokens.
 // Algorithmic bytes: B*N*(T*elt + 12) read + B*fh*fw*T*elt written.
 #include <algorithm>
 
 #include "avits_common.cuh"
 #include "avits_internal.h"
+#include "frame_map.cuh"
 
 namespace avits {
 namespace {
@@ -274,10 +275,6 @@ merge_nearest_kernel(const T* __restrict__ mixed, int B, int N, const int32_t* _
   if (twice) raise_status(status, AVITS_ERR_COVERAGE);   // a cell claimed twice
 }
 
-// Cell map entry: the covering token's index, with kSpan2 set when its span
-// is 2 (the gather then needs no span lookup); -1 = a hole.
-constexpr int32_t kSpan2 = 1 << 30;
-
 // The cell map starts as -1 everywhere (a hole until a token claims it).
 __global__ void merge_fill_kernel(int32_t* __restrict__ map, int64_t n) {
   pdl_wait_then_trigger();
@@ -286,6 +283,7 @@ __global__ void merge_fill_kernel(int32_t* __restrict__ map, int64_t n) {
     map[i] = -1;
 }
 
+// One thread per token: its s x s cells get map_entry(token, log2 s).
 __global__ void merge_map_kernel(int B, int N, const int32_t* __restrict__ pos,
                                  const int32_t* __restrict__ span, int fh, int fw,
                                  int32_t* __restrict__ map, unsigned int* status) {
@@ -294,12 +292,12 @@ __global__ void merge_map_kernel(int B, int N, const int32_t* __restrict__ pos,
   if (t >= (int64_t)B * N) return;
   const int b = (int)(t / N), ti = (int)(t % N);
   const int y = pos[t * 2], x = pos[t * 2 + 1], s = span[t];
-  if ((s != 1 && s != 2) || y < 0 || x < 0 || y + s > fh || x + s > fw ||
-      (s == 2 && ((y | x) & 1))) {
+  const int lvl = (s == 1) ? 0 : (s == 2) ? 1 : (s == 4) ? 2 : -1;
+  if (lvl < 0 || y < 0 || x < 0 || y + s > fh || x + s > fw || ((y | x) & (s - 1))) {
     raise_status(status, AVITS_ERR_COVERAGE);
     return;
   }
-  const int32_t entry = ti | (s == 2 ? kSpan2 : 0);
+  const int32_t entry = map_entry(ti, lvl);
   for (int u = 0; u < s; ++u)
     for (int v = 0; v < s; ++v) {
       const int old = atomicExch(&map[(int64_t)b * fh * fw + (int64_t)(y + u) * fw + x + v], entry);
@@ -307,35 +305,17 @@ __global__ void merge_map_kernel(int B, int N, const int32_t* __restrict__ pos,
     }
 }
 
-// Low-resolution pixel (r, c) of the rebuilt grid from the map entries of its
-// even-aligned cell (e0) and of its own cell (e1): a span-2 token gives its
-// patch pixel, a span-1 token its 2x2 average pool ((a+b)+(c+d))/4; 0 for a
-// hole (already reported).
+// One thread per (output cell, channel).  A span-1 cell is copied.  A coarser
+// cell's four pixels are the 2x bilinear resize of level 1 around it (a 3 x 3
+// neighbourhood of level-1 pixels, clamped to the frame), where level 1 is the
+// frame's own pyramid level, or, inside a span-4 token, the 2x bilinear
+// resize of level 2 (the coarse-to-fine cascade; spans are at most 4).
 template <typename T>
-__device__ __forceinline__ float low_value(const T* __restrict__ mb, int T4, int ch, int r, int c,
-                                           int32_t e0, int32_t e1) {
-  if (e0 < 0) return 0.f;
-  if (e0 & kSpan2)
-    return load_elem(mb, (int64_t)(e0 & ~kSpan2) * T4 + ch * 4 + (r & 1) * 2 + (c & 1));
-  if (e1 < 0) return 0.f;
-  const T* p = mb + (int64_t)(e1 & ~kSpan2) * T4 + ch * 4;
-  const float top = __fadd_rn(load_elem(p, 0), load_elem(p, 1));
-  const float bot = __fadd_rn(load_elem(p, 2), load_elem(p, 3));
-  return __fmul_rn(__fadd_rn(top, bot), 0.25f);
-}
-
-// One thread per (output cell, channel).  A span-2 cell's four pixels draw on
-// the 3 x 3 low-resolution neighbourhood around it; all map entries of that
-// neighbourhood are loaded first, then all pixel values, so the chains of
-// dependent loads are two deep.
-template <typename T>
-__global__ void merge_bilinear_kernel(const T* __restrict__ mixed, int B, int N,
-                                      const int32_t* __restrict__ span, int fh, int fw, int C,
-                                      const int32_t* __restrict__ map, T* __restrict__ out,
+__global__ void merge_bilinear_kernel(const T* __restrict__ mixed, int B, int N, int fh, int fw,
+                                      int C, const int32_t* __restrict__ map, T* __restrict__ out,
                                       unsigned int* status) {
   using PV = typename Pix4<T>::V;
   pdl_wait_then_trigger();
-  (void)span;
   const int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t cells = (int64_t)fh * fw;
   if (g >= (int64_t)B * cells * C) return;
@@ -354,44 +334,39 @@ __global__ void merge_bilinear_kernel(const T* __restrict__ mixed, int B, int N,
     *dst = Pix4<T>::make(0.f, 0.f, 0.f, 0.f);
     return;
   }
-  if (!(e & kSpan2)) {
-    *dst = reinterpret_cast<const PV*>(mb + (int64_t)e * T4)[c];
+  if (map_lvl(e) == 0) {
+    *dst = reinterpret_cast<const PV*>(mb + (int64_t)map_tok(e) * T4)[c];
     return;
   }
-  // rows and columns of the neighbourhood (clamped to the frame)
+  // level-1 pixels (rows Y-1..Y+1, columns X-1..X+1, clamped): the frame's
+  // own, or inside a span-4 token the resize of level 2
   int rr[3], cc[3];
 #pragma unroll
   for (int k = 0; k < 3; ++k) {
     rr[k] = min(max(Y - 1 + k, 0), fh - 1);
     cc[k] = min(max(X - 1 + k, 0), fw - 1);
   }
-  int32_t e0[3][3], e1[3][3];
-#pragma unroll
-  for (int i = 0; i < 3; ++i)
-#pragma unroll
-    for (int j = 0; j < 3; ++j) {
-      e0[i][j] = mapb[(rr[i] & ~1) * fw + (cc[j] & ~1)];
-      e1[i][j] = mapb[rr[i] * fw + cc[j]];
-    }
   float lv[3][3];
 #pragma unroll
   for (int i = 0; i < 3; ++i)
 #pragma unroll
-    for (int j = 0; j < 3; ++j) lv[i][j] = low_value(mb, T4, c, rr[i], cc[j], e0[i][j], e1[i][j]);
+    for (int j = 0; j < 3; ++j) {
+      const int32_t en = mapb[(int64_t)rr[i] * fw + cc[j]];
+      lv[i][j] = (en >= 0 && map_lvl(en) >= 2)
+                     ? frame_resize2x(2, mb, T4, mapb, fh, fw, c, rr[i], cc[j])
+                     : frame_pixel<1>(mb, T4, mapb, fw, c, rr[i], cc[j]);
+    }
   float r[4];
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
-    // output pixel row 2Y + a draws on rows (Y - 1, Y) for a = 0 and (Y, Y + 1)
-    // for a = 1 with weights (1/4, 3/4) / (3/4, 1/4), clamped at the frame
-    // edge: neighbourhood rows a and a + 1; columns likewise
+    // output pixel row 2Y + a draws on level-1 rows (Y - 1, Y) for a = 0 and
+    // (Y, Y + 1) for a = 1 with weights (1/4, 3/4) / (3/4, 1/4), clamped at
+    // the frame edge: neighbourhood rows a and a + 1; columns likewise
     const int a = q >> 1, bq = q & 1;
     const float wy0 = a ? 0.75f : 0.25f, wy1 = a ? 0.25f : 0.75f;
     const float wx0 = bq ? 0.75f : 0.25f, wx1 = bq ? 0.25f : 0.75f;
-    const float p00 = lv[a][bq], p01 = lv[a][bq + 1];
-    const float p10 = lv[a + 1][bq], p11 = lv[a + 1][bq + 1];
-    const float top = __fadd_rn(__fmul_rn(wx0, p00), __fmul_rn(wx1, p01));
-    const float bot = __fadd_rn(__fmul_rn(wx0, p10), __fmul_rn(wx1, p11));
-    r[q] = __fadd_rn(__fmul_rn(wy0, top), __fmul_rn(wy1, bot));
+    r[q] = bil_combine(lv[a][bq], lv[a][bq + 1], lv[a + 1][bq], lv[a + 1][bq + 1], wy0, wy1, wx0,
+                       wx1);
   }
   *dst = Pix4<T>::make(r[0], r[1], r[2], r[3]);
 }
@@ -432,10 +407,24 @@ cudaError_t launch_t(const void* mixed, int B, int N, const int32_t* pos, const 
   // programmatic dependent of the one before: their launches overlap, every
   // kernel waits for its predecessor before touching memory
   int32_t* map = reinterpret_cast<int32_t*>(words);
+  cudaError_t e = launch_cell_map(B, N, pos, span, fh, fw, map, status, s);
+  if (e == cudaSuccess) e = prefer_max_shared<merge_bilinear_kernel<T>>();
+  if (e != cudaSuccess) return e;
+  const int64_t work = (int64_t)B * fh * fw * C;
+  e = launch_pdl(merge_bilinear_kernel<T>, dim3((unsigned)((work + 255) / 256)), dim3(256), 0, s,
+                 static_cast<const T*>(mixed), B, N, fh, fw, C,
+                 static_cast<const int32_t*>(map), static_cast<T*>(out), status);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_cell_map(int B, int N, const int32_t* pos, const int32_t* span, int fh, int fw,
+                            int32_t* map, unsigned int* status, cudaStream_t s) {
   const int64_t ncell = (int64_t)B * fh * fw;
   cudaError_t e = prefer_max_shared<merge_fill_kernel>();
   if (e == cudaSuccess) e = prefer_max_shared<merge_map_kernel>();
-  if (e == cudaSuccess) e = prefer_max_shared<merge_bilinear_kernel<T>>();
   if (e != cudaSuccess) return e;
   const int fill_grid = (int)std::min<int64_t>((ncell + 255) / 256, 1024);
   e = launch_pdl(merge_fill_kernel, dim3(fill_grid), dim3(256), 0, s, map, ncell);
@@ -444,15 +433,8 @@ cudaError_t launch_t(const void* mixed, int B, int N, const int32_t* pos, const 
   e = launch_pdl(merge_map_kernel, dim3((unsigned)((nt + 255) / 256)), dim3(256), 0, s, B, N, pos,
                  span, fh, fw, map, status);
   if (e != cudaSuccess) return e;
-  const int64_t work = (int64_t)B * fh * fw * C;
-  e = launch_pdl(merge_bilinear_kernel<T>, dim3((unsigned)((work + 255) / 256)), dim3(256), 0, s,
-                 static_cast<const T*>(mixed), B, N, span, fh, fw, C,
-                 static_cast<const int32_t*>(map), static_cast<T*>(out), status);
-  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
-
-}  // namespace
 
 size_t merge_workspace_bytes(int B, int fh, int fw) {
   return kMergeHeaderBytes + sizeof(uint32_t) * (size_t)B * fh * fw;

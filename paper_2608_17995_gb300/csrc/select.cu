@@ -699,14 +699,16 @@ cudaError_t launch_select_upsample(const float* A, const float* V, const float* 
                                    int gh, int gw, int C, const int32_t* pos_in,
                                    const int32_t* span_in, avits_upmode mode, void* out,
                                    int32_t* out_pos, int32_t* out_span, int32_t* out_src_tok,
-                                   int8_t* out_src_sub, cudaStream_t s) {
-  if (M > kFusedMaxM) {
-    // beyond one CTA's registers: the two launches, same outputs
+                                   int8_t* out_src_sub, void* ws, cudaStream_t s) {
+  if (M > kFusedMaxM || (mode == AVITS_UP_BILINEAR && pos_in)) {
+    // beyond one CTA's registers, or a mixed bilinear input (whose cell map
+    // is built between the selection and the upsample): the separate
+    // launches, same outputs
     cudaError_t e = launch_fuse_select(A, V, perturb, B, M, alpha, eps, k, S, sel_idx, mask,
                                        tok_offset, status, s);
     if (e != cudaSuccess) return e;
     return launch_upsample(latent, dt, B, M, gh, gw, C, pos_in, span_in, mask, tok_offset, k,
-                           mode, out, out_pos, out_span, out_src_tok, out_src_sub, s);
+                           mode, out, out_pos, out_span, out_src_tok, out_src_sub, ws, status, s);
   }
   const SelArgs g{A, V, perturb, M, alpha, eps, k, S, sel_idx, mask, tok_offset, status};
   if (dt == AVITS_BF16)

@@ -8,7 +8,9 @@
 //                the 2x upsample of the parent's pixel (a,b): nearest
 //                broadcasts the pixel; bilinear applies the fixed 0.25 / 0.75
 //                weights of a half-pixel-centred 2x resize with edge clamping,
-//                reading neighbouring pixels from the dense input latent.
+//                reading neighbouring pixels from the dense input latent, or,
+//                for a mixed input, from level log2(s) of the input frame's
+//                pixel pyramid through its cell map (frame_map.cuh).
 // Nearest with 16-byte token rows: each lane writes whole 16-byte chunks
 // (coalesced); otherwise lanes split the (child, channel) work, each writing
 // the 4 pixels of one channel of one child.  Lanes 0-3 write the position /
@@ -16,24 +18,9 @@
 #pragma once
 
 #include "avits_common.cuh"
+#include "frame_map.cuh"
 
 namespace avits {
-
-__device__ __forceinline__ void bil_axis(int P, int n, int& r0, int& r1, float& w0, float& w1) {
-  const int m = P >> 1;
-  if ((P & 1) == 0) { r0 = m - 1; r1 = m; w0 = 0.25f; w1 = 0.75f; }
-  else { r0 = m; r1 = m + 1; w0 = 0.75f; w1 = 0.25f; }
-  r0 = max(r0, 0);
-  r1 = min(r1, n - 1);
-}
-
-// wy0*(wx0*p00 + wx1*p01) + wy1*(wx0*p10 + wx1*p11), rounded step by step
-__device__ __forceinline__ float bil_combine(float p00, float p01, float p10, float p11,
-                                            float wy0, float wy1, float wx0, float wx1) {
-  const float top = __fadd_rn(__fmul_rn(wx0, p00), __fmul_rn(wx1, p01));
-  const float bot = __fadd_rn(__fmul_rn(wx0, p10), __fmul_rn(wx1, p11));
-  return __fadd_rn(__fmul_rn(wy0, top), __fmul_rn(wy1, bot));
-}
 
 template <typename T>
 struct UpsampleArgs {
@@ -46,6 +33,9 @@ struct UpsampleArgs {
   int32_t* out_span;               // [B,n_out]
   int32_t* out_src_tok;            // [B,n_out]
   int8_t* out_src_sub;             // [B,n_out]
+  // bilinear with a mixed input: the input frame's cell map [B,gh,gw]
+  // (frame_map.cuh); NULL for a dense grid
+  const int32_t* map = nullptr;
 };
 
 // Where a token's C*4 source values are read from: element b's rows of the
@@ -110,11 +100,28 @@ __device__ __forceinline__ void upsample_token(const UpsampleArgs<T>& u, const S
     const PV* sp = reinterpret_cast<const PV*>(src);
     for (int c = lane; c < C; c += 32) dst[c] = sp[c];
   } else {
+    // a mixed input token of span 2^l is resized from level l of the input
+    // frame's pyramid; an invalid position or span (reported by the map
+    // kernel) gives zeros
+    const int lv = (s == 1) ? 0 : (s == 2) ? 1 : (s == 4) ? 2 : -1;
+    const bool frame_ok = lv >= 0 && y >= 0 && x >= 0 && y + s <= gh && x + s <= gw &&
+                          ((y | x) & (s - 1)) == 0;
     for (int task = lane; task < 4 * C; task += 32) {
       const int child = task / C, c = task - child * C;
       const int a = child >> 1, bb = child & 1;
       PV v;
-      if (!kBilinear) {
+      if (kBilinear && u.map) {
+        float r[4] = {0.f, 0.f, 0.f, 0.f};
+        if (frame_ok) {
+          const T* tokb = u.latent + (int64_t)b * M * T4;
+          const int32_t* mapb = u.map + (int64_t)b * gh * gw;
+          const int R0 = 2 * ((2 * y) >> lv) + 2 * a, Q0 = 2 * ((2 * x) >> lv) + 2 * bb;
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            r[q] = frame_resize2x(lv, tokb, T4, mapb, gh, gw, c, R0 + (q >> 1), Q0 + (q & 1));
+        }
+        v = Pix4<T>::make(r[0], r[1], r[2], r[3]);
+      } else if (!kBilinear) {
         const float p = load_elem(src, c * 4 + a * 2 + bb);
         v = Pix4<T>::make(p, p, p, p);
       } else {

@@ -11,7 +11,8 @@ import numpy as np
 
 from . import (BILINEAR, NEAREST, SpatialWorkspace, avits_fuse_select, avits_merge_final,
                avits_merge_final_workspace, avits_score_spatial, avits_score_spatiotemporal,
-               avits_score_temporal, avits_select_upsample, avits_selective_upsample)
+               avits_score_temporal, avits_select_upsample, avits_selective_upsample,
+               avits_selective_upsample_workspace)
 
 
 def to_device(arr: np.ndarray, dtype: str, device="cuda"):
@@ -70,6 +71,9 @@ class TransitionBuffers:
         mb = avits_merge_final_workspace(self.mode, B, self.full_h, self.full_w)
         # zero-filled before first use (the nearest merge's claim map and counter)
         self.merge_ws = torch.zeros(max(mb, 16), dtype=torch.uint8, **z) if mb else None
+        # a mixed input in bilinear mode: the input frame's cell map
+        ub = avits_selective_upsample_workspace(self.mode, B, tr.frame_h, tr.frame_w)
+        self.up_ws = torch.empty(ub, dtype=torch.uint8, **z) if ub else None
 
     def set_inputs(self, q, k, h_t, h_prev, latent, pos_in=None, span_in=None):
         self.q, self.k, self.h_t, self.h_prev, self.latent = q, k, h_t, h_prev, latent
@@ -97,7 +101,7 @@ class TransitionBuffers:
         avits_selective_upsample(self.latent, self.tr.frame_h, self.tr.frame_w, self.sel_mask,
                                  self.tok_offset, self.tr.k, self.mixed, self.pos, self.span,
                                  self.src_tok, self.src_sub, mode=self.mode, pos_in=self.pos_in,
-                                 span_in=self.span_in, stream=stream)
+                                 span_in=self.span_in, workspace=self.up_ws, stream=stream)
 
     def select_upsample(self, stream=None):
         """Selection and selective upsampling in one launch."""
@@ -105,7 +109,7 @@ class TransitionBuffers:
                               self.tok_offset, self.sel_mask, self.latent, self.tr.frame_h,
                               self.tr.frame_w, self.mixed, self.pos, self.span, self.src_tok,
                               self.src_sub, S=self.S, mode=self.mode, pos_in=self.pos_in,
-                              span_in=self.span_in, stream=stream)
+                              span_in=self.span_in, workspace=self.up_ws, stream=stream)
 
     def merge(self, stream=None):
         avits_merge_final(self.mixed, self.pos, self.span, self.full_h, self.full_w, self.full,

@@ -814,3 +814,118 @@ def test_batched_two_transitions(av, orc):
     full_o, cover = orc.merge_final(o[0], o[1], o[2], 64, 64)
     assert np.all(cover == 1)
     assert np.array_equal(_bits(_np(b2.full)), _bits(full_o))
+
+
+# ------------------------------------------- multi-level bilinear (spans 1, 2, 4)
+
+def test_batched_two_transitions_bilinear(av, orc):
+    """The batched schedule in bilinear mode: the second transition upsamples
+    selected span-1 and span-2 tokens from levels 0 and 1 of the mixed
+    frame's pyramid, and the final merge (spans 1, 2 and 4) runs the
+    coarse-to-fine cascade; both bit-exact against the oracle (given the
+    kernel's own selection, itself checked against the oracle's top-k)."""
+    from paper_2608_17995_gb300.pipeline import TransitionBuffers
+    from paper_2608_17995_gb300.workloads import make_batched_stage2, make_transition
+    t1 = make_transition("batched")
+    b1 = TransitionBuffers(t1, mode="bilinear")
+    b1.run(merge=False)
+    assert _status(av) == 0
+    mixed1, pos1, span1 = _np(b1.mixed), _np(b1.pos), _np(b1.span)
+    _, mask1_o, _ = orc.topk(_np(b1.S), t1.k)
+    o1 = orc.selective_upsample(t1.latent, 16, 16, mask1_o, mode="bilinear")
+    assert np.array_equal(_bits(mixed1), _bits(o1[0]))
+    t2 = make_batched_stage2(pos1, span1, frame=32, latent=mixed1)
+    b2 = TransitionBuffers(t2, mode="bilinear")
+    b2.run()
+    assert _status(av) == 0
+    _, mask_o, _ = orc.topk(_np(b2.S), t2.k)
+    assert np.array_equal(_np(b2.sel_mask), mask_o)
+    o = orc.selective_upsample(mixed1, 32, 32, mask_o, mode="bilinear", pos_in=pos1,
+                               span_in=span1)
+    assert set(np.unique(o[2])) == {1, 2, 4}
+    assert np.array_equal(_bits(_np(b2.mixed)), _bits(o[0]))
+    assert np.array_equal(_np(b2.pos), o[1]) and np.array_equal(_np(b2.span), o[2])
+    full_o, cover = orc.merge_final(o[0], o[1], o[2], 64, 64, mode="bilinear")
+    assert np.all(cover == 1)
+    assert np.array_equal(_bits(_np(b2.full)), _bits(full_o))
+
+
+@pytest.mark.parametrize("dtype,case", [("f32", "random"), ("bf16", "random"),
+                                        ("f32", "all"), ("bf16", "none"), ("f32", "none-all")])
+def test_multilevel_bilinear_bit_exact(av, orc, dtype, case):
+    """Two transitions in bilinear mode on a 12x10 grid (ragged frame, C = 6):
+    random selections (spans 1, 2 and 4 mixed), everything selected, nothing
+    selected (span-4 merge), nothing then everything; the second upsample
+    through both entry points (avits_selective_upsample and the selection +
+    upsample call, which routes a mixed bilinear input through the cell
+    map) and the merge, bit-exact against the oracle."""
+    import torch
+    from paper_2608_17995_gb300.workloads import random_scores, to_bf16_bits
+    B, gh, gw, C = 2, 12, 10, 6
+    M = gh * gw
+    lat = np.random.default_rng(31).standard_normal((B, M, 4 * C)).astype(np.float32)
+    if dtype == "bf16":
+        lat = to_bf16_bits(lat)
+    k1 = {"random": 30, "all": M, "none": 0, "none-all": 0}[case]
+    _, m1, off1 = orc.topk(random_scores(41, B, M)[0], k1)
+    g1 = _upsample(av, lat, dtype, gh, gw, m1, off1, k1, 1)
+    o1 = orc.selective_upsample(lat, gh, gw, m1, mode="bilinear")
+    assert np.array_equal(_bits(g1[0]), _bits(o1[0]))
+    N1 = o1[0].shape[1]
+    k2 = {"random": 70, "all": N1, "none": 0, "none-all": N1}[case]
+    A2, V2 = random_scores(42, B, N1)
+    S2 = orc.fuse(A2, V2, 0.5)
+    _, m2, off2 = orc.topk(S2, k2)
+    g2 = _upsample(av, o1[0], dtype, 2 * gh, 2 * gw, m2, off2, k2, 1, pos_in=o1[1],
+                   span_in=o1[2])
+    o2 = orc.selective_upsample(o1[0], 2 * gh, 2 * gw, m2, mode="bilinear", pos_in=o1[1],
+                                span_in=o1[2])
+    for a, b in zip(g2, o2):
+        assert np.array_equal(_bits(a) if a.dtype.kind == "f" or a.dtype == np.uint16 else a,
+                              _bits(b) if b.dtype.kind == "f" or b.dtype == np.uint16 else b)
+    # the selection + upsample entry point on the same mixed input
+    tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    NO = N1 + 3 * k2
+    outs = [torch.full((B, NO, 4 * C), float("nan"), dtype=tdt, device="cuda"),
+            torch.zeros(B, NO, 2, dtype=torch.int32, device="cuda"),
+            torch.zeros(B, NO, dtype=torch.int32, device="cuda"),
+            torch.zeros(B, NO, dtype=torch.int32, device="cuda"),
+            torch.zeros(B, NO, dtype=torch.int8, device="cuda")]
+    sel = torch.zeros(B, max(k2, 1), dtype=torch.int32, device="cuda")
+    off = torch.zeros(B, N1, dtype=torch.int32, device="cuda")
+    msk = torch.zeros(B, N1, dtype=torch.uint8, device="cuda")
+    av.avits_select_upsample(_dev(A2), _dev(V2), 0.5, k2, sel, off, msk, _dev(o1[0], dtype),
+                             2 * gh, 2 * gw, *outs, mode=1, pos_in=_dev(o1[1]),
+                             span_in=_dev(o1[2]))
+    assert _status(av) == 0
+    assert np.array_equal(_np(msk), m2)
+    assert np.array_equal(_bits(_np(outs[0])), _bits(o2[0]))
+    assert np.array_equal(_np(outs[1]), o2[1]) and np.array_equal(_np(outs[2]), o2[2])
+    if case == "none":
+        assert np.all(o2[2] == 4)
+    full_g = _merge(av, o2[0], dtype, o2[1], o2[2], 4 * gh, 4 * gw, 1)
+    full_o, _ = orc.merge_final(o2[0], o2[1], o2[2], 4 * gh, 4 * gw, mode="bilinear")
+    assert np.array_equal(_bits(full_g), _bits(full_o))
+
+
+def test_multilevel_bilinear_rejects_other_spans(av, orc):
+    """Spans outside {1, 2, 4} (or off their alignment) in a bilinear merge or
+    a mixed bilinear upsample raise AVITS_ERR_COVERAGE on the device; the
+    next valid call is clean."""
+    import torch
+    lat = np.random.default_rng(2).standard_normal((1, 4, 8)).astype(np.float32)
+    out, pos, span, _, _ = orc.selective_upsample(lat, 2, 2, np.zeros((1, 4), np.uint8))
+    # one span-8 token over the whole 8x8 frame
+    big = np.zeros((1, 1, 8), np.float32)
+    _merge(av, big, "f32", np.zeros((1, 1, 2), np.int32), np.full((1, 1), 8, np.int32), 8, 8, 1,
+           expect_status=6)
+    _merge(av, out, "f32", pos, span, 4, 4, 1)
+    # a mixed upsample input whose span-2 token sits off its alignment
+    bad = pos.copy()
+    bad[0, 1] = (0, 1)
+    mask = np.ones((1, 4), np.uint8)
+    _, _, off = orc.topk(np.ones((1, 4), np.float32), 4)
+    with pytest.raises(AssertionError):
+        _upsample(av, out, "f32", 4, 4, mask, off, 4, 1, pos_in=bad, span_in=span)
+    assert _status(av) == 0
+    _upsample(av, out, "f32", 4, 4, mask, off, 4, 1, pos_in=pos, span_in=span)

@@ -58,8 +58,9 @@ def test_host_validation_rejects_without_launch(lib):
     assert lib.avits_score_temporal(P, P, 1, 1, 0, 64, 1e-6, P, None) == INVALID
     snaps = (ctypes.c_void_p * 17)(*([16] * 17))
     assert lib.avits_score_temporal_var(snaps, 17, 1, 1, 4, 8, P, None) == INVALID
-    # upsample: patch size other than 2, grid that does not match M, bilinear on mixed input
-    up = [P, 1, 1, 16, 4, 4, 16, 2, None, None, P, P, 4, 0, P, P, P, P, P, None]
+    # upsample: patch size other than 2, grid that does not match M; a mixed
+    # input in bilinear mode needs the cell-map workspace and an even frame
+    up = [P, 1, 1, 16, 4, 4, 16, 2, None, None, P, P, 4, 0, P, P, P, P, P, None, 0, None]
     up[7] = 3
     assert lib.avits_selective_upsample(*up) == UNSUPPORTED
     up[7] = 2
@@ -67,7 +68,15 @@ def test_host_validation_rejects_without_launch(lib):
     assert lib.avits_selective_upsample(*up) == INVALID
     up[4] = 4
     up[8], up[9], up[13] = P, P, 1
-    assert lib.avits_selective_upsample(*up) == UNSUPPORTED
+    assert lib.avits_selective_upsample(*up) == INVALID          # no workspace
+    wsb = lib.avits_selective_upsample_workspace(1, 1, 4, 4)
+    assert wsb == 16 + 4 * 16
+    assert lib.avits_selective_upsample_workspace(0, 1, 4, 4) == 0
+    up[19], up[20] = P, wsb - 4
+    assert lib.avits_selective_upsample(*up) == INVALID          # too small
+    up[20] = wsb
+    up[4], up[5] = 3, 5                                           # odd frame
+    assert lib.avits_selective_upsample(*up) == INVALID
     # merge: both modes need a workspace (16-byte aligned, large enough);
     # bilinear an even frame; misaligned output
     mg = [P, 1, 1, 28, P, P, 8, 8, 1, 2, 1, P, None, 0, None]
@@ -128,9 +137,9 @@ def test_host_validation_of_the_extended_entry_points(lib):
     km[15] = 0.0
     assert lib.avits_score_spatial_keymask(*km) == INVALID
     # fused selection + upsample: the mask is required, k > M, patch size
-    # other than 2, bilinear on mixed-level input
+    # other than 2, bilinear on mixed-level input without its workspace
     su = [P, P, None, 1, 16, 0.5, 1e-6, 4, None, P, None, P, P, 1, 4, 4, 16, 2, None, None, 0,
-          P, P, P, P, P, None]
+          P, P, P, P, P, None, 0, None]
     assert lib.avits_select_upsample(*su) == INVALID
     su[10] = P
     su[7] = 17
@@ -140,7 +149,7 @@ def test_host_validation_of_the_extended_entry_points(lib):
     assert lib.avits_select_upsample(*su) == UNSUPPORTED
     su[17] = 2
     su[18], su[19], su[20] = P, P, 1
-    assert lib.avits_select_upsample(*su) == UNSUPPORTED
+    assert lib.avits_select_upsample(*su) == INVALID
 
 
 def test_host_validation_of_the_wait_selftest(lib):
