@@ -15,32 +15,36 @@
 // runs over all key tiles (128 keys), so O and the row statistics stay in
 // the CTA and no partial results cross CTAs (except Eq. 3's head sum).
 //
-// Tensor memory (512 columns): S_t / P_t of query tile t at columns
-// [128t, 128t + 128), O_t at [256 + Dt, 256 + D(t+1)).  P_t (bf16 pairs)
-// overwrites the first 64 columns of S_t, each 16-column block after the
-// softmax has read the 32 S columns it replaces.
+// Tensor memory (512 columns): S_t of query tile t at columns [128t, 128t +
+// 128), O_t at [256 + Dt, 256 + D(t+1)).  P goes through shared memory, so
+// that S_t is free as soon as the softmax has loaded it: the next key tile's
+// S_t = Q_t K^T then runs on the tensor pipe while the softmax computes the
+// exponentials of this one.
 //
 // Roles (12 warps):
-//   warp 0       TMA producer: Q tile 0, K_0, Q tile 1, V_0, then K_j, V_j
-//                through a ring of 128-key tiles (128-byte swizzle).
+//   warp 0       TMA producer: Q tiles, then the K and V tiles through a
+//                3-stage ring in the order the MMAs consume them (K_0, K_1,
+//                V_0, K_2, V_1, ...), 128-byte swizzle.
 //   warps 1, 2   MMA issuers of query tile 0 / 1 (warp 1 owns tensor
-//                memory): per key tile S_t = Q_t K_j^T (tcgen05.mma, both
-//                operands K-major in shared memory), then, once the softmax
-//                has written P_t, O_t += P_t V_j (A = P_t from tensor memory,
-//                B = V_j as an MN-major shared-memory operand, no transpose
-//                copy).  S_t of the next key tile overwrites P_t, so it is
-//                issued when that PV product has completed; the other tile's
-//                issuer keeps the tensor pipe busy meanwhile.
+//                memory): for key tile g, S_t(g) = Q_t K_g^T once the softmax
+//                has loaded S_t(g-1), then O_t += P_t(g-1) V_(g-1) once that P
+//                is in shared memory.  Both products are tcgen05.mma kind::f16
+//                from shared memory; V is read in its natural [keys, d] layout
+//                as an MN-major operand (no transpose copy).
 //   warp 3       no role.
 //   warps 4-7    softmax and epilogue of query tile 0, warps 8-11 of tile 1:
-//                one row per thread (TMEM lane), two passes over the 128 S
-//                columns of an item (row maximum, then exponentials, sums and
-//                P).  The running maximum is raised only when a key tile's
-//                maximum exceeds it by more than 2^8 (P <= 256 otherwise, no
-//                loss in bf16 or the fp32 accumulator); then l and O are
-//                rescaled in place.  The epilogue divides O by the row sum,
-//                stages it in shared memory in the TMA's swizzled layout and
-//                stores it with one bulk tensor copy per 64 columns.
+//                one row per thread (TMEM lane); the row's 128 S columns are loaded into registers and
+//                S_t released; the row maximum; the running maximum is raised
+//                only when a key tile's maximum exceeds it by more than 2^8
+//                (P <= 256 otherwise, no loss in bf16 or the fp32
+//                accumulator), and then l and O are rescaled (O in tensor
+//                memory, by the whole warp); the exponentials (packed FMA +
+//                MUFU), the fp32 sums over all keys and over the text keys
+//                (the only addition the score needs) and the bf16 P row, written
+//                to shared memory in the K-major 128-byte-swizzled layout the
+//                MMA reads.  The epilogue divides O by the row sum, stages it
+//                in the P buffer and stores it with one bulk tensor copy per 64
+//                columns.
 // Every wait is bounded (avits_common.cuh); after a timeout every role skips
 // its remaining work, drains what it issued and the CTA releases tensor
 // memory and exits.
@@ -71,24 +75,26 @@ struct Cfg {
   static constexpr int kStages = (D == 128) ? 3 : 6;   // K / V ring
   static constexpr int kQBytes = kQTiles * kTileBytes;
   static constexpr int kKVBytes = kStages * kTileBytes;
-  static constexpr int kOBytes = kQTiles * kTileBytes; // O staging, one tile each
   static constexpr uint32_t kIdescPV = idesc_bf16(kBM, D, true);
 };
+// P of one query tile: 128 rows x 128 keys bf16 (two 128-byte column blocks);
+// at a unit's end the same buffer stages that tile's O (D <= 128 columns)
+constexpr int kPTileBytes = 2 * kBM * 128;
+constexpr int kPBytes = kQTiles * kPTileBytes;
 constexpr int kMaxStages = 6;
 
 struct Bars {
   uint64_t q_full[kQTiles], q_empty[kQTiles];
   uint64_t kv_full[kMaxStages], kv_empty[kMaxStages];
-  uint64_t s_full[kQTiles], p_full[kQTiles], pv_done[kQTiles];
+  uint64_t s_full[kQTiles], s_empty[kQTiles], p_full[kQTiles], pv_done[kQTiles];
   uint64_t o_full[kQTiles], o_empty[kQTiles], drain[kQTiles];
-  uint64_t t1_go;   // one phase: tile 0's first P is written
   uint32_t tmem_base;
   int abort;
 };
 
 template <int D>
 constexpr int smem_bytes() {
-  return Cfg<D>::kQBytes + Cfg<D>::kKVBytes + Cfg<D>::kOBytes + (int)sizeof(Bars) + 1024;
+  return Cfg<D>::kQBytes + Cfg<D>::kKVBytes + kPBytes + (int)sizeof(Bars) + 1024;
 }
 
 struct AttnParams {
@@ -117,11 +123,6 @@ __device__ __forceinline__ bool bar_and(int id, int count, bool v) {
   return r != 0;
 }
 
-__device__ __forceinline__ void wait_ld2(uint32_t (&a)[32], uint32_t (&b)[32]) {
-  tmem_wait32(a);
-  tmem_wait32(b);   // already complete; ties b's registers to the wait
-}
-
 // Row maximum of 32 S columns whose first key is col0; keys >= Nk are left
 // out (kFull: all 32 are valid).
 template <bool kFull>
@@ -143,146 +144,77 @@ __device__ __forceinline__ float chunk_max(const uint32_t (&r)[32], int col0, in
   return fmaxf(max3(u0, u1, u2), fmaxf(t[9], t[10]));
 }
 
-// Exponentials of 32 S columns (first key col0) against the running maximum
-// m: their fp32 sum (all keys, text keys) and the bf16 P words for tensor
-// memory.  kKind: 0 = valid image keys, 1 = valid text keys, 2 = general
-// (keys beyond Nk give 0, text keys counted one by one).
-template <int kKind>
-__device__ __forceinline__ void chunk_exp(const uint32_t (&r)[32], int col0, int Nk, int L,
-                                          float c, float m, float& la, float& lt,
-                                          uint32_t (&w)[16]) {
-  const float nm = -m;
-  float p[32];
-#pragma unroll
-  for (int e = 0; e < 32; e += 2) {
-    float x0, x1;
-    ffma2(__uint_as_float(r[e]), __uint_as_float(r[e + 1]), c, nm, x0, x1);
-    p[e] = ex2(x0);
-    p[e + 1] = ex2(x1);
-  }
-  if (kKind == 2) {
-#pragma unroll
-    for (int e = 0; e < 32; ++e)
-      if (col0 + e >= Nk) p[e] = 0.f;
-  }
-  float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-#pragma unroll
-  for (int e = 0; e < 32; e += 4) {
-    fadd2(s0, s1, p[e], p[e + 1]);
-    fadd2(s2, s3, p[e + 2], p[e + 3]);
-  }
-  fadd2(s0, s1, s2, s3);
-  const float cs = s0 + s1;
-  la += cs;
-  if (kKind == 1) {
-    lt += cs;
-  } else if (kKind == 2 && col0 < L) {
-    float ts = 0.f;
-#pragma unroll
-    for (int e = 0; e < 32; ++e) ts += (col0 + e < L) ? p[e] : 0.f;
-    lt += ts;
-  }
-#pragma unroll
-  for (int e = 0; e < 16; ++e) w[e] = pack_bf16x2(p[2 * e], p[2 * e + 1]);
-}
-
-// Kind of the 32 keys starting at col0 (uniform over the warp).
-__device__ __forceinline__ int chunk_kind(int col0, int Nk, int L) {
-  if (col0 + 32 <= Nk) {
-    if (col0 + 32 <= L) return 1;
-    if (col0 >= L) return 0;
-  }
-  return 2;
-}
-
-__device__ __forceinline__ void exp_by_kind(int kind, const uint32_t (&r)[32], int col0, int Nk,
-                                            int L, float c, float m, float& la, float& lt,
-                                            uint32_t (&w)[16]) {
-  if (kind == 0)
-    chunk_exp<0>(r, col0, Nk, L, c, m, la, lt, w);
-  else if (kind == 1)
-    chunk_exp<1>(r, col0, Nk, L, c, m, la, lt, w);
-  else
-    chunk_exp<2>(r, col0, Nk, L, c, m, la, lt, w);
-}
-
-// O_t row *= f (D fp32 columns at tO).
+// O_t row *= f (D fp32 columns at tO), 16 columns at a time.
 template <int D>
 __device__ __forceinline__ void rescale_o(uint32_t tO, float f) {
 #pragma unroll 1
-  for (int k = 0; k < D / 32; ++k) {
-    uint32_t r[32];
-    tmem_ld32(tO + 32 * k, r);
-    tmem_wait32(r);
+  for (int k = 0; k < D / 16; ++k) {
+    uint32_t r[16];
+    tmem_ld16(tO + 16 * k, r);
+    tmem_wait(r);
 #pragma unroll
-    for (int e = 0; e < 32; e += 2) {
+    for (int e = 0; e < 16; e += 2) {
       float a0 = __uint_as_float(r[e]), a1 = __uint_as_float(r[e + 1]);
       fmul2(a0, a1, f);
       r[e] = __float_as_uint(a0);
       r[e + 1] = __float_as_uint(a1);
     }
-    tmem_st32(tO + 32 * k, r);
+    tmem_st16(tO + 16 * k, r);
   }
+}
+
+// Exponentials of 32 S columns (first key col0) against the running maximum
+// m, their fp32 sums (all keys, text keys) and the bf16 P values, stored as
+// four 16-byte chunks of the row's P block: chunk q (keys col0 + 8q ..) at
+// position (jj0 + q) ^ (row & 7) of the 128-byte row (the K-major 128-byte
+// swizzle).  Eight columns at a time, so few values are live besides r.
+// kKind: 0 = valid image keys, 1 = valid text keys, 2 = general (keys beyond
+// Nk give 0, text keys counted one by one).
+template <int kKind>
+__device__ __forceinline__ void emit_chunk(const uint32_t (&r)[32], int col0, int Nk, int L,
+                                           float c, float m, float& la, float& lt,
+                                           uint8_t* rowp, int jj0, int rsw) {
+  const float nm = -m;
+  float s0 = 0.f, s1 = 0.f, t0 = 0.f;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    float e[8];
+#pragma unroll
+    for (int i = 0; i < 8; i += 2) {
+      float x0, x1;
+      ffma2(__uint_as_float(r[8 * q + i]), __uint_as_float(r[8 * q + i + 1]), c, nm, x0, x1);
+      e[i] = ex2(x0);
+      e[i + 1] = ex2(x1);
+    }
+    if (kKind == 2) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        if (col0 + 8 * q + i >= Nk) e[i] = 0.f;
+        if (col0 + 8 * q + i < L) t0 += e[i];
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 8; i += 2) fadd2(s0, s1, e[i], e[i + 1]);
+    *reinterpret_cast<uint4*>(rowp + (((jj0 + q) ^ rsw) << 4)) =
+        make_uint4(pack_bf16x2(e[0], e[1]), pack_bf16x2(e[2], e[3]), pack_bf16x2(e[4], e[5]),
+                   pack_bf16x2(e[6], e[7]));
+  }
+  const float cs = s0 + s1;
+  la += cs;
+  if (kKind == 1) lt += cs;
+  if (kKind == 2) lt += t0;
 }
 
 struct RowState {
   float m, la, lt;
 };
 
-// One key tile of one row: S at tS (128 fp32 columns), P written to the
-// first 64 columns, the running statistics updated, O rescaled when the
-// maximum moves.  first: the row's first key tile of the unit (O holds no
-// sum yet).
-template <int D>
-__device__ __forceinline__ void softmax_item(uint32_t tS, uint32_t tO, int key0, int Nk, int L,
-                                             float c, bool first, RowState& st) {
-  uint32_t ra[32], rb[32];
-  const bool full = key0 + kBN <= Nk;
-  // pass 1: the tile's row maximum
-  tmem_ld32(tS, ra);
-  tmem_ld32(tS + 32, rb);
-  wait_ld2(ra, rb);
-  float mx = full ? fmaxf(chunk_max<true>(ra, 0, 0), chunk_max<true>(rb, 0, 0))
-                  : fmaxf(chunk_max<false>(ra, key0, Nk), chunk_max<false>(rb, key0 + 32, Nk));
-  tmem_ld32(tS + 64, ra);
-  tmem_ld32(tS + 96, rb);
-  wait_ld2(ra, rb);
-  mx = full ? fmaxf(mx, fmaxf(chunk_max<true>(ra, 0, 0), chunk_max<true>(rb, 0, 0)))
-            : fmaxf(mx, fmaxf(chunk_max<false>(ra, key0 + 64, Nk),
-                              chunk_max<false>(rb, key0 + 96, Nk)));
-  const float mt = mx * c;
-  const bool up = mt > st.m + kTau;   // the row's first tile, or a logit 2^8 above its maximum
-  float f = 1.f;
-  if (up) {
-    f = ex2(st.m - mt);
-    st.la *= f;
-    st.lt *= f;
-    st.m = mt;
-  }
-  // tcgen05.ld / st are warp-collective: the warp rescales its O rows
-  // together when any of them moved (f = 1 leaves a row unchanged)
-  if (!first && __any_sync(0xffffffffu, up)) rescale_o<D>(tO, f);
-  // pass 2: exponentials, sums and P, 32 columns at a time; P block k
-  // (columns [16k, 16k + 16)) replaces S columns already read
-  uint32_t w[16];
-  tmem_ld32(tS, ra);
-  tmem_wait32(ra);
-  tmem_ld32(tS + 32, rb);
-  exp_by_kind(chunk_kind(key0, Nk, L), ra, key0, Nk, L, c, st.m, st.la, st.lt, w);
-  tmem_st16(tS, w);
-  tmem_wait32(rb);
-  tmem_ld32(tS + 64, ra);
-  exp_by_kind(chunk_kind(key0 + 32, Nk, L), rb, key0 + 32, Nk, L, c, st.m, st.la, st.lt, w);
-  tmem_st16(tS + 16, w);
-  tmem_wait32(ra);
-  tmem_ld32(tS + 96, rb);
-  exp_by_kind(chunk_kind(key0 + 64, Nk, L), ra, key0 + 64, Nk, L, c, st.m, st.la, st.lt, w);
-  tmem_st16(tS + 32, w);
-  tmem_wait32(rb);
-  exp_by_kind(chunk_kind(key0 + 96, Nk, L), rb, key0 + 96, Nk, L, c, st.m, st.la, st.lt, w);
-  tmem_st16(tS + 48, w);
-  tmem_wait_st();
-}
+// Indices of a key tile's K and V loads in the ring: the load order is the
+// order the MMAs consume them, K_0, K_1, V_0, K_2, V_1, ... (S of the next
+// key tile is issued before P V of this one).  The K slot after the last
+// key tile is left unused.
+__device__ __forceinline__ int k_load(int g) { return g == 0 ? 0 : 2 * g - 1; }
+__device__ __forceinline__ int v_load(int g) { return 2 * g + 2; }
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -295,12 +227,13 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sQ = smem;
   uint8_t* sKV = sQ + C::kQBytes;
-  uint8_t* sO = sKV + C::kKVBytes;
-  Bars* bars = reinterpret_cast<Bars*>(sO + C::kOBytes);
+  uint8_t* sP = sKV + C::kKVBytes;   // P of each query tile; the O staging at a unit's end
+  Bars* bars = reinterpret_cast<Bars*>(sP + kPBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n_my = (p.n_units - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
   if (n_my <= 0) return;   // block-uniform
+  const int G = n_my * p.n_kt;   // key tiles this CTA processes (all its units)
 
   if (threadIdx.x == 0) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQ)) : "memory");
@@ -311,13 +244,13 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
       mbar_init(&bars->q_full[t], 1);
       mbar_init(&bars->q_empty[t], 1);
       mbar_init(&bars->s_full[t], 1);
-      mbar_init(&bars->p_full[t], 4);     // the tile's 4 softmax warps
+      mbar_init(&bars->s_empty[t], 4);    // the tile's 4 softmax warps
+      mbar_init(&bars->p_full[t], 4);
       mbar_init(&bars->pv_done[t], 1);
       mbar_init(&bars->o_full[t], 1);
       mbar_init(&bars->o_empty[t], 4);
       mbar_init(&bars->drain[t], 1);
     }
-    mbar_init(&bars->t1_go, 4);
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&bars->kv_full[s], 1);
       mbar_init(&bars->kv_empty[s], kQTiles);   // one commit per issuer
@@ -347,110 +280,118 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
     // ------------------------------------------------------ TMA producer --
     if (lane == 0) {
       bool ok = true;
-      int li = 0;        // ring loads issued (K and V tiles)
-      int q_armed = 0;   // Q tiles of the current unit issued
-      int ui = 0;
-      for (; ui < n_my && ok; ++ui) {
+      int last[C::kStages];   // the latest load armed on each stage, -1 = none
+      for (int s = 0; s < C::kStages; ++s) last[s] = -1;
+      int q_armed = 0, q_unit = 0;   // Q tiles armed for unit q_unit
+      auto load_q = [&](int ui, int t) {
         int b, h, qp;
         unit_coords((int)blockIdx.x + ui * (int)gridDim.x, b, h, qp);
-        q_armed = 0;
-        auto load_q = [&](int t) {
-          if (ui > 0) ok = mbar_wait_bounded(&bars->q_empty[t], (uint32_t)((ui - 1) & 1), abort_flag, p.status);
-          if (!ok) return;
-          mbar_arrive_expect_tx(&bars->q_full[t], C::kTileBytes);
-          for (int cb = 0; cb < C::kCB; ++cb)
-            tma_load_4d(sQ + t * C::kTileBytes + cb * (kBM * 128), &tmQ, cb * 64,
-                        qp * kUnitRows + t * kBM, h, b, &bars->q_full[t]);
-          ++q_armed;
-        };
-        auto load_kv = [&](const CUtensorMap* map, int kt) {
-          const int stage = li % C::kStages;
-          const uint32_t ph = (uint32_t)((li / C::kStages) & 1);
-          ok = mbar_wait_bounded(&bars->kv_empty[stage], ph ^ 1u, abort_flag, p.status);
-          if (!ok) return;
-          mbar_arrive_expect_tx(&bars->kv_full[stage], C::kTileBytes);
-          for (int cb = 0; cb < C::kCB; ++cb)
-            tma_load_4d(sKV + stage * C::kTileBytes + cb * (kBM * 128), map, cb * 64, kt * kBN, h,
-                        b, &bars->kv_full[stage]);
-          ++li;
-        };
-        load_q(0);
-        if (ok) load_kv(&tmK, 0);
-        if (ok) load_q(1);
-        for (int j = 0; j < p.n_kt && ok; ++j) {
-          load_kv(&tmV, j);
-          if (ok && j + 1 < p.n_kt) load_kv(&tmK, j + 1);
+        if (ui > 0)
+          ok = mbar_wait_bounded(&bars->q_empty[t], (uint32_t)((ui - 1) & 1), abort_flag, p.status);
+        if (!ok) return;
+        if (q_unit != ui) { q_unit = ui; q_armed = 0; }
+        mbar_arrive_expect_tx(&bars->q_full[t], C::kTileBytes);
+        for (int cb = 0; cb < C::kCB; ++cb)
+          tma_load_4d(sQ + t * C::kTileBytes + cb * (kBM * 128), &tmQ, cb * 64,
+                      qp * kUnitRows + t * kBM, h, b, &bars->q_full[t]);
+        ++q_armed;
+      };
+      // load number idx of the ring: key tile g's K (is_k) or V
+      auto load_kv = [&](int idx, bool is_k, int g) {
+        int b, h, qp;
+        unit_coords((int)blockIdx.x + (g / p.n_kt) * (int)gridDim.x, b, h, qp);
+        const int kt = g - (g / p.n_kt) * p.n_kt;
+        const int stage = idx % C::kStages;
+        const uint32_t ph = (uint32_t)((idx / C::kStages) & 1);
+        ok = mbar_wait_bounded(&bars->kv_empty[stage], ph ^ 1u, abort_flag, p.status);
+        if (!ok) return;
+        mbar_arrive_expect_tx(&bars->kv_full[stage], C::kTileBytes);
+        for (int cb = 0; cb < C::kCB; ++cb)
+          tma_load_4d(sKV + stage * C::kTileBytes + cb * (kBM * 128), is_k ? &tmK : &tmV, cb * 64,
+                      kt * kBN, h, b, &bars->kv_full[stage]);
+        last[stage] = idx;
+      };
+      load_q(0, 0);
+      if (ok) load_kv(k_load(0), true, 0);
+      if (ok) load_q(0, 1);
+      for (int g = 0; g < G && ok; ++g) {
+        const int gn = g + 1;
+        if (gn < G) {
+          if (gn % p.n_kt == 0) {   // the next unit's Q tiles before its first K tile
+            load_q(gn / p.n_kt, 0);
+            if (ok) load_q(gn / p.n_kt, 1);
+          }
+          if (ok) load_kv(k_load(gn), true, gn);
         }
+        if (ok) load_kv(v_load(g), false, g);
       }
       if (!ok) {
-        // drain the copies still in flight: the Q tiles of the last unit
-        // started, then the last load of every ring stage
-        const int ul = ui - 1;
+        // drain the copies still in flight before the CTA exits
         for (int t = 0; t < q_armed; ++t)
-          mbar_wait_bounded(&bars->q_full[t], (uint32_t)(ul & 1), nullptr, p.status);
-        for (int s = 0; s < C::kStages; ++s) {
-          const int armed = li - s;   // loads issued on stage s: li - s > 0
-          if (armed > 0) {
-            const int last = (armed - 1) / C::kStages;
-            mbar_wait_bounded(&bars->kv_full[s], (uint32_t)(last & 1), nullptr, p.status);
-          }
-        }
+          mbar_wait_bounded(&bars->q_full[t], (uint32_t)(q_unit & 1), nullptr, p.status);
+        for (int s = 0; s < C::kStages; ++s)
+          if (last[s] >= 0)
+            mbar_wait_bounded(&bars->kv_full[s], (uint32_t)((last[s] / C::kStages) & 1), nullptr,
+                              p.status);
       }
     }
   } else if (warp == 1 || warp == 2) {
     // -------------------------------------------------------- MMA issuers --
+    // Key tile g: S_t(g) = Q_t K_g^T as soon as the softmax has loaded
+    // S_t(g-1); then O_t += P_t(g-1) V_(g-1) once P_t(g-1) is in shared
+    // memory.  The tensor pipe so holds the next S while the softmax works.
     const int t = warp - 1;
     if (lane == 0) {
       bool ok = true;
-      int gi = 0;   // key tiles processed by this CTA (all units)
-      const uint32_t a_lo = sw128_desc_lo(sQ + t * C::kTileBytes);
+      const uint32_t q_lo = sw128_desc_lo(sQ + t * C::kTileBytes);
+      const uint32_t p_lo = sw128_desc_lo(sP + t * kPTileBytes);
       const uint32_t kv_lo0 = sw128_desc_lo(sKV);
       const uint32_t v_lo0 = sw128_mn_desc_lo(sKV, kBM * 128);
       const uint32_t d_hi = sw128_desc_hi();
       const uint32_t tS = tmem + (uint32_t)(t * kBN);
       const uint32_t tO = tmem + (uint32_t)(2 * kBN + t * D);
-      for (int ui = 0; ui < n_my && ok; ++ui) {
-        for (int j = 0; j < p.n_kt && ok; ++j, ++gi) {
-          // S_t = Q_t K_j^T
-          const int lk = 2 * gi, lv = 2 * gi + 1;
-          const int sk = lk % C::kStages, sv = lv % C::kStages;
+      for (int gi = 0; gi <= G && ok; ++gi) {
+        if (gi < G) {
+          const int ui = gi / p.n_kt, j = gi - ui * p.n_kt;
+          const int lk = k_load(gi), sk = lk % C::kStages;
           ok = mbar_wait_bounded(&bars->kv_full[sk], (uint32_t)((lk / C::kStages) & 1), abort_flag, p.status);
           if (ok && j == 0)
             ok = mbar_wait_bounded(&bars->q_full[t], (uint32_t)(ui & 1), abort_flag, p.status);
-          // tile 1 starts one softmax behind tile 0, so that the two tiles'
-          // S, softmax and PV stages overlap instead of running in lockstep
-          if (ok && t == 1 && gi == 0)
-            ok = mbar_wait_bounded(&bars->t1_go, 0u, abort_flag, p.status);
-          // P_t of the previous key tile has been read by its PV product
-          if (ok && gi > 0)
-            ok = mbar_wait_bounded(&bars->pv_done[t], (uint32_t)((gi - 1) & 1), abort_flag, p.status);
+          if (ok && gi > 0)   // the softmax has loaded S_t(gi - 1)
+            ok = mbar_wait_bounded(&bars->s_empty[t], (uint32_t)((gi - 1) & 1), abort_flag, p.status);
           if (!ok) break;
           fence_after();
           const uint32_t k_lo = kv_lo0 + (uint32_t)((sk * C::kTileBytes) >> 4);
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
             const uint32_t off = (uint32_t)(((kk >> 2) * (kBM * 128) + (kk & 3) * 32) >> 4);
-            mma_ss(tS, a_lo + off, k_lo + off, d_hi, kIdescS, kk > 0 ? 1u : 0u);
+            mma_ss(tS, q_lo + off, k_lo + off, d_hi, kIdescS, kk > 0 ? 1u : 0u);
           }
           mma_commit(&bars->s_full[t]);
           mma_commit(&bars->kv_empty[sk]);
           if (j == p.n_kt - 1) mma_commit(&bars->q_empty[t]);
-          // O_t += P_t V_j
-          ok = mbar_wait_bounded(&bars->p_full[t], (uint32_t)(gi & 1), abort_flag, p.status);
+        }
+        if (gi > 0) {
+          const int g = gi - 1;
+          const int ug = g / p.n_kt, jg = g - ug * p.n_kt;
+          const int lv = v_load(g), sv = lv % C::kStages;
+          ok = mbar_wait_bounded(&bars->p_full[t], (uint32_t)(g & 1), abort_flag, p.status);
           if (ok)
             ok = mbar_wait_bounded(&bars->kv_full[sv], (uint32_t)((lv / C::kStages) & 1), abort_flag, p.status);
-          if (ok && j == 0 && ui > 0)   // the epilogue has read the previous unit's O_t
-            ok = mbar_wait_bounded(&bars->o_empty[t], (uint32_t)((ui - 1) & 1), abort_flag, p.status);
+          if (ok && jg == 0 && ug > 0)   // the epilogue has read the previous unit's O_t
+            ok = mbar_wait_bounded(&bars->o_empty[t], (uint32_t)((ug - 1) & 1), abort_flag, p.status);
           if (!ok) break;
           fence_after();
           const uint32_t v_lo = v_lo0 + (uint32_t)((sv * C::kTileBytes) >> 4);
 #pragma unroll
-          for (int kk = 0; kk < kBN / 16; ++kk)   // 16 keys: 8 P columns, 16 V rows
-            mma_ts(tO, tS + (uint32_t)(kk * 8), v_lo + (uint32_t)((kk * 16 * 128) >> 4), d_hi,
-                   C::kIdescPV, (j > 0 || kk > 0) ? 1u : 0u);
+          for (int kk = 0; kk < kBN / 16; ++kk) {   // 16 keys: 16 P columns, 16 V rows
+            const uint32_t off = (uint32_t)(((kk >> 2) * (kBM * 128) + (kk & 3) * 32) >> 4);
+            mma_ss(tO, p_lo + off, v_lo + (uint32_t)((kk * 16 * 128) >> 4), d_hi, C::kIdescPV,
+                   (jg > 0 || kk > 0) ? 1u : 0u);
+          }
           mma_commit(&bars->pv_done[t]);
           mma_commit(&bars->kv_empty[sv]);
-          if (j == p.n_kt - 1) mma_commit(&bars->o_full[t]);
+          if (jg == p.n_kt - 1) mma_commit(&bars->o_full[t]);
         }
       }
       // all issued MMAs complete before tensor memory is released
@@ -467,7 +408,8 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
     const uint32_t tS = tmem + lane_off + (uint32_t)(t * kBN);
     const uint32_t tO = tmem + lane_off + (uint32_t)(2 * kBN + t * D);
-    uint8_t* stg = sO + t * C::kTileBytes;
+    uint8_t* sPt = sP + t * kPTileBytes;
+    const float c = p.c_log2;
     bool ok = true;
     int gi = 0;
     for (int ui = 0; ui < n_my; ++ui) {
@@ -480,21 +422,85 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
         ok = __all_sync(0xffffffffu, ok);   // tcgen05.ld / st are warp-collective
         if (ok) {
           fence_after();
-          softmax_item<D>(tS, tO, j * kBN, p.Nk, p.L, p.c_log2, j == 0, st);
+          // the row's 128 S columns into registers; S_t is then free for the
+          // next key tile's MMA
+          uint32_t r0[32], r1[32], r2[32], r3[32];
+          tmem_ld32(tS, r0);
+          tmem_ld32(tS + 32, r1);
+          tmem_ld32(tS + 64, r2);
+          tmem_ld32(tS + 96, r3);
+          tmem_wait32(r0);
+          tmem_wait32(r1);
+          tmem_wait32(r2);
+          tmem_wait32(r3);
           fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bars->s_empty[t]);
+          const int key0 = j * kBN;
+          float mx;
+          if (key0 + kBN <= p.Nk)
+            mx = fmaxf(fmaxf(chunk_max<true>(r0, 0, 0), chunk_max<true>(r1, 0, 0)),
+                       fmaxf(chunk_max<true>(r2, 0, 0), chunk_max<true>(r3, 0, 0)));
+          else
+            mx = fmaxf(fmaxf(chunk_max<false>(r0, key0, p.Nk), chunk_max<false>(r1, key0 + 32, p.Nk)),
+                       fmaxf(chunk_max<false>(r2, key0 + 64, p.Nk),
+                             chunk_max<false>(r3, key0 + 96, p.Nk)));
+          const float mt = mx * c;
+          const bool up = mt > st.m + kTau;   // the row's first tile, or 2^8 above its maximum
+          float f = 1.f;
+          if (up) {
+            f = ex2(st.m - mt);
+            st.la *= f;
+            st.lt *= f;
+            st.m = mt;
+          }
+          // P_t(gi - 1) has been read by its PV product and O_t holds it
+          if (gi > 0) {
+            bool w = mbar_wait_bounded(&bars->pv_done[t], (uint32_t)((gi - 1) & 1), abort_flag, p.status);
+            ok = __all_sync(0xffffffffu, w);
+          }
+          if (ok) {
+            // exponentials, sums and the bf16 P row into shared memory (K-major,
+            // 128-byte swizzle: 16-byte chunk q of the row's block at q ^ (row & 7))
+            // the kind is uniform over the warp: one branch per key tile
+            // for the whole-image and whole-text tiles, per chunk otherwise
+            uint8_t* rowp0 = sPt + rowt * 128;
+            uint8_t* rowp1 = rowp0 + kBM * 128;
+            const int rsw = rowt & 7;
+            if (key0 + kBN <= p.Nk && key0 >= p.L) {
+              emit_chunk<0>(r0, key0, p.Nk, p.L, c, st.m, st.la, st.lt, rowp0, 0, rsw);
+              emit_chunk<0>(r1, key0 + 32, p.Nk, p.L, c, st.m, st.la, st.lt, rowp0, 4, rsw);
+              emit_chunk<0>(r2, key0 + 64, p.Nk, p.L, c, st.m, st.la, st.lt, rowp1, 0, rsw);
+              emit_chunk<0>(r3, key0 + 96, p.Nk, p.L, c, st.m, st.la, st.lt, rowp1, 4, rsw);
+            } else if (key0 + kBN <= p.Nk && key0 + kBN <= p.L) {
+              emit_chunk<1>(r0, key0, p.Nk, p.L, c, st.m, st.la, st.lt, rowp0, 0, rsw);
+              emit_chunk<1>(r1, key0 + 32, p.Nk, p.L, c, st.m, st.la, st.lt, rowp0, 4, rsw);
+              emit_chunk<1>(r2, key0 + 64, p.Nk, p.L, c, st.m, st.la, st.lt, rowp1, 0, rsw);
+              emit_chunk<1>(r3, key0 + 96, p.Nk, p.L, c, st.m, st.la, st.lt, rowp1, 4, rsw);
+            } else {
+              emit_chunk<2>(r0, key0, p.Nk, p.L, c, st.m, st.la, st.lt, rowp0, 0, rsw);
+              emit_chunk<2>(r1, key0 + 32, p.Nk, p.L, c, st.m, st.la, st.lt, rowp0, 4, rsw);
+              emit_chunk<2>(r2, key0 + 64, p.Nk, p.L, c, st.m, st.la, st.lt, rowp1, 0, rsw);
+              emit_chunk<2>(r3, key0 + 96, p.Nk, p.L, c, st.m, st.la, st.lt, rowp1, 4, rsw);
+            }
+            // the warp rescales its O rows together when any of them moved
+            // (f = 1 leaves a row unchanged)
+            if (j > 0 && __any_sync(0xffffffffu, up)) {
+              rescale_o<D>(tO, f);
+              tmem_wait_st();
+            }
+            fence_async_shared();   // P is read by the tensor core (async proxy)
+            fence_before();
+          }
         }
         __syncwarp();
-        if (ok && lane == 0) {
-          mbar_arrive(&bars->p_full[t]);
-          if (t == 0 && gi == 0) mbar_arrive(&bars->t1_go);
-        }
+        if (ok && lane == 0) mbar_arrive(&bars->p_full[t]);
       }
-      // ---- epilogue: O / l -> bf16 -> swizzled staging -> TMA store
+      // ---- epilogue: O / l -> bf16 -> swizzled staging (the P buffer, free
+      // once the last PV product completed) -> TMA store
       ok = ok && (*abort_flag == 0) &&
            mbar_wait_bounded(&bars->o_full[t], (uint32_t)(ui & 1), abort_flag, p.status);
       ok = __all_sync(0xffffffffu, ok);
-      if (leader) bulk_wait_read();   // the previous unit's store has read the staging tile
-      bar_sync(bar_id, 128);
       if (ok) {
         fence_after();
         const float inv = 1.f / st.la;
@@ -507,11 +513,9 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
 #pragma unroll
           for (int e = 0; e < 16; ++e)
             w[e] = pack_bf16x2(__uint_as_float(r[2 * e]) * inv, __uint_as_float(r[2 * e + 1]) * inv);
-          // columns [32k, 32k + 32): block cb, 16-byte chunks jj .. jj + 3 of
-          // the row, each at chunk (jj ^ row) of the 128-byte swizzle
           const int cb = (32 * k) >> 6;
           const int jj0 = ((32 * k) & 63) >> 3;
-          uint8_t* rowp = stg + cb * (kBM * 128) + rowt * 128;
+          uint8_t* rowp = sPt + cb * (kBM * 128) + rowt * 128;
 #pragma unroll
           for (int q = 0; q < 4; ++q)
             *reinterpret_cast<uint4*>(rowp + (((jj0 + q) ^ (rowt & 7)) << 4)) =
@@ -537,9 +541,11 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
       const bool all_ok = bar_and(bar_id, 128, ok);
       if (all_ok && leader && qp * kUnitRows + t * kBM < p.Mq) {   // a tile past the end stores nothing
         for (int cb = 0; cb < C::kCB; ++cb)
-          tma_store_4d(&tmO, stg + cb * (kBM * 128), cb * 64, qp * kUnitRows + t * kBM, h, b);
+          tma_store_4d(&tmO, sPt + cb * (kBM * 128), cb * 64, qp * kUnitRows + t * kBM, h, b);
         bulk_commit();
+        bulk_wait_read();   // the staging is the next unit's P buffer
       }
+      bar_sync(bar_id, 128);
     }
     if (leader) bulk_wait_all();
   }
