@@ -164,45 +164,58 @@ __device__ __forceinline__ void rescale_o(uint32_t tO, float f) {
 }
 
 // Exponentials of 32 S columns (first key col0) against the running maximum
-// m, their fp32 sums (all keys, text keys) and the bf16 P values, stored as
-// four 16-byte chunks of the row's P block: chunk q (keys col0 + 8q ..) at
-// position (jj0 + q) ^ (row & 7) of the 128-byte row (the K-major 128-byte
-// swizzle).  Eight columns at a time, so few values are live besides r.
-// kKind: 0 = valid image keys, 1 = valid text keys, 2 = general (keys beyond
-// Nk give 0, text keys counted one by one).
+// m, in place (r then holds the fp32 softmax numerators), and their fp32 sums
+// over all keys and over the text keys.  kKind: 0 = valid image keys, 1 =
+// valid text keys, 2 = general (keys beyond Nk give 0, text keys counted one
+// by one).
 template <int kKind>
-__device__ __forceinline__ void emit_chunk(const uint32_t (&r)[32], int col0, int Nk, int L,
-                                           float c, float m, float& la, float& lt,
-                                           uint8_t* rowp, int jj0, int rsw) {
+__device__ __forceinline__ void exp_chunk(uint32_t (&r)[32], int col0, int Nk, int L, float c,
+                                          float m, float& la, float& lt) {
   const float nm = -m;
   float s0 = 0.f, s1 = 0.f, t0 = 0.f;
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    float e[8];
-#pragma unroll
-    for (int i = 0; i < 8; i += 2) {
-      float x0, x1;
-      ffma2(__uint_as_float(r[8 * q + i]), __uint_as_float(r[8 * q + i + 1]), c, nm, x0, x1);
-      e[i] = ex2(x0);
-      e[i + 1] = ex2(x1);
-    }
+  for (int e = 0; e < 32; e += 2) {
+    float x0, x1;
+    ffma2(__uint_as_float(r[e]), __uint_as_float(r[e + 1]), c, nm, x0, x1);
+    float e0 = ex2(x0), e1 = ex2(x1);
     if (kKind == 2) {
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        if (col0 + 8 * q + i >= Nk) e[i] = 0.f;
-        if (col0 + 8 * q + i < L) t0 += e[i];
-      }
+      if (col0 + e >= Nk) e0 = 0.f;
+      if (col0 + e + 1 >= Nk) e1 = 0.f;
+      if (col0 + e < L) t0 += e0;
+      if (col0 + e + 1 < L) t0 += e1;
     }
-#pragma unroll
-    for (int i = 0; i < 8; i += 2) fadd2(s0, s1, e[i], e[i + 1]);
-    *reinterpret_cast<uint4*>(rowp + (((jj0 + q) ^ rsw) << 4)) =
-        make_uint4(pack_bf16x2(e[0], e[1]), pack_bf16x2(e[2], e[3]), pack_bf16x2(e[4], e[5]),
-                   pack_bf16x2(e[6], e[7]));
+    fadd2(s0, s1, e0, e1);
+    r[e] = __float_as_uint(e0);
+    r[e + 1] = __float_as_uint(e1);
   }
   const float cs = s0 + s1;
   la += cs;
   if (kKind == 1) lt += cs;
   if (kKind == 2) lt += t0;
+}
+
+template <int kKind>
+__device__ __forceinline__ void exp_tile(uint32_t (&r0)[32], uint32_t (&r1)[32],
+                                         uint32_t (&r2)[32], uint32_t (&r3)[32], int key0,
+                                         int Nk, int L, float c, float m, float& la, float& lt) {
+  exp_chunk<kKind>(r0, key0, Nk, L, c, m, la, lt);
+  exp_chunk<kKind>(r1, key0 + 32, Nk, L, c, m, la, lt);
+  exp_chunk<kKind>(r2, key0 + 64, Nk, L, c, m, la, lt);
+  exp_chunk<kKind>(r3, key0 + 96, Nk, L, c, m, la, lt);
+}
+
+// 32 fp32 numerators -> bf16, four 16-byte chunks of the row's P block: chunk
+// q at position (jj0 + q) ^ (row & 7) of the 128-byte row (the K-major
+// 128-byte swizzle the MMA reads).
+__device__ __forceinline__ void store_p(const uint32_t (&r)[32], uint8_t* rowp, int jj0, int rsw) {
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    *reinterpret_cast<uint4*>(rowp + (((jj0 + q) ^ rsw) << 4)) =
+        make_uint4(pack_bf16x2(__uint_as_float(r[8 * q]), __uint_as_float(r[8 * q + 1])),
+                   pack_bf16x2(__uint_as_float(r[8 * q + 2]), __uint_as_float(r[8 * q + 3])),
+                   pack_bf16x2(__uint_as_float(r[8 * q + 4]), __uint_as_float(r[8 * q + 5])),
+                   pack_bf16x2(__uint_as_float(r[8 * q + 6]), __uint_as_float(r[8 * q + 7])));
+  }
 }
 
 struct RowState {
@@ -454,35 +467,27 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
             st.lt *= f;
             st.m = mt;
           }
+          // the numerators in place while the previous PV product may still
+          // be reading the P buffer; the kind is uniform over the warp
+          if (key0 + kBN <= p.Nk && key0 >= p.L)
+            exp_tile<0>(r0, r1, r2, r3, key0, p.Nk, p.L, c, st.m, st.la, st.lt);
+          else if (key0 + kBN <= p.Nk && key0 + kBN <= p.L)
+            exp_tile<1>(r0, r1, r2, r3, key0, p.Nk, p.L, c, st.m, st.la, st.lt);
+          else
+            exp_tile<2>(r0, r1, r2, r3, key0, p.Nk, p.L, c, st.m, st.la, st.lt);
           // P_t(gi - 1) has been read by its PV product and O_t holds it
           if (gi > 0) {
             bool w = mbar_wait_bounded(&bars->pv_done[t], (uint32_t)((gi - 1) & 1), abort_flag, p.status);
             ok = __all_sync(0xffffffffu, w);
           }
           if (ok) {
-            // exponentials, sums and the bf16 P row into shared memory (K-major,
-            // 128-byte swizzle: 16-byte chunk q of the row's block at q ^ (row & 7))
-            // the kind is uniform over the warp: one branch per key tile
-            // for the whole-image and whole-text tiles, per chunk otherwise
             uint8_t* rowp0 = sPt + rowt * 128;
             uint8_t* rowp1 = rowp0 + kBM * 128;
             const int rsw = rowt & 7;
-            if (key0 + kBN <= p.Nk && key0 >= p.L) {
-              emit_chunk<0>(r0, key0, p.Nk, p.L, c, st.m, st.la, st.lt, rowp0, 0, rsw);
-              emit_chunk<0>(r1, key0 + 32, p.Nk, p.L, c, st.m, st.la, st.lt, rowp0, 4, rsw);
-              emit_chunk<0>(r2, key0 + 64, p.Nk, p.L, c, st.m, st.la, st.lt, rowp1, 0, rsw);
-              emit_chunk<0>(r3, key0 + 96, p.Nk, p.L, c, st.m, st.la, st.lt, rowp1, 4, rsw);
-            } else if (key0 + kBN <= p.Nk && key0 + kBN <= p.L) {
-              emit_chunk<1>(r0, key0, p.Nk, p.L, c, st.m, st.la, st.lt, rowp0, 0, rsw);
-              emit_chunk<1>(r1, key0 + 32, p.Nk, p.L, c, st.m, st.la, st.lt, rowp0, 4, rsw);
-              emit_chunk<1>(r2, key0 + 64, p.Nk, p.L, c, st.m, st.la, st.lt, rowp1, 0, rsw);
-              emit_chunk<1>(r3, key0 + 96, p.Nk, p.L, c, st.m, st.la, st.lt, rowp1, 4, rsw);
-            } else {
-              emit_chunk<2>(r0, key0, p.Nk, p.L, c, st.m, st.la, st.lt, rowp0, 0, rsw);
-              emit_chunk<2>(r1, key0 + 32, p.Nk, p.L, c, st.m, st.la, st.lt, rowp0, 4, rsw);
-              emit_chunk<2>(r2, key0 + 64, p.Nk, p.L, c, st.m, st.la, st.lt, rowp1, 0, rsw);
-              emit_chunk<2>(r3, key0 + 96, p.Nk, p.L, c, st.m, st.la, st.lt, rowp1, 4, rsw);
-            }
+            store_p(r0, rowp0, 0, rsw);
+            store_p(r1, rowp0, 4, rsw);
+            store_p(r2, rowp1, 0, rsw);
+            store_p(r3, rowp1, 4, rsw);
             // the warp rescales its O rows together when any of them moved
             // (f = 1 leaves a row unchanged)
             if (j > 0 && __any_sync(0xffffffffu, up)) {
