@@ -117,7 +117,7 @@ avits_status avits_score_spatial(const void* q_img, const void* k_all, avits_dty
     return cuda_status(launch_spatial_tc(a, sms, s));
   }
   if (d > 256) return AVITS_ERR_UNSUPPORTED;
-  return cuda_status(launch_spatial_simt(a, s));
+  return cuda_status(launch_spatial_simt(a, num_sms_current(), s));
 }
 
 avits_status avits_score_spatial_lse(const void* q_img, const void* k_txt, avits_dtype dt, int B,
@@ -167,7 +167,7 @@ avits_status avits_score_spatial_keymask(const void* q_img, const void* k_all, a
     return cuda_status(launch_spatial_tc(a, sms, s));
   }
   if (d > 256) return AVITS_ERR_UNSUPPORTED;
-  return cuda_status(launch_spatial_simt(a, s));
+  return cuda_status(launch_spatial_simt(a, num_sms_current(), s));
 }
 
 size_t avits_attention_forward_workspace(int B, int H, int Mq) {
@@ -259,7 +259,7 @@ avits_status avits_score_spatiotemporal(const void* q_img, const void* k_all, av
     return cuda_status(launch_spatial_tc(a, sms, s, &temporal));
   }
   if (d > 256) return AVITS_ERR_UNSUPPORTED;
-  cudaError_t e = launch_spatial_simt(a, s);
+  cudaError_t e = launch_spatial_simt(a, num_sms_current(), s);
   if (e == cudaSuccess) e = launch_temporal(h_t, h_prev, dt, B, M, D, eps, V, sms, a.status, s);
   return cuda_status(e);
 }

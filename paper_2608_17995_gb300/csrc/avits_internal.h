@@ -67,8 +67,8 @@ using LaunchHook = std::function<cudaError_t(cudaStream_t)>;
 cudaError_t launch_spatial_tc(const SpatialArgs& a, int num_sms, cudaStream_t s,
                               const LaunchHook* between = nullptr);
 
-// CUDA-core path (fp32 or bf16, any d <= 256): one warp per query row.
-cudaError_t launch_spatial_simt(const SpatialArgs& a, cudaStream_t s);
+// CUDA-core path (fp32 or bf16, any d <= 256): up to 8 query rows per CTA.
+cudaError_t launch_spatial_simt(const SpatialArgs& a, int num_sms, cudaStream_t s);
 
 // ---- joint-attention forward (Eq. 4-5) with the spatial score (Eq. 3) -------
 struct AttnArgs {
