@@ -371,6 +371,9 @@ avits_status avits_fuse_select_perturbed(const float* A, const float* V, const f
  *          contents (the call rebuilds the frame's cell map there); otherwise
  *          ignored (may be NULL).
  * sel_mask, tok_offset : from avits_fuse_select.  k = number selected.
+ *          A token whose outputs would not lie inside [0, M+3k) (tok_offset
+ *          < 0, or above M+3k-4 for a selected / M+3k-1 for a deferred token)
+ *          is not written and raises AVITS_ERR_COVERAGE on the device.
  * out_latent : [B,M+3k,C*4] same dtype.  out_pos : [B,M+3k,2] (row, col).
  * out_span : [B,M+3k].  out_src_tok : [B,M+3k] input token index.
  * out_src_sub : [B,M+3k] int8, child number 0..3, or -1 for a deferred token.

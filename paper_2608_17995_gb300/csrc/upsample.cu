@@ -22,7 +22,8 @@ upsample_kernel(const T* __restrict__ latent, int B, int M, int gh, int gw, int 
                 const uint8_t* __restrict__ mask, const int32_t* __restrict__ tok_offset,
                 int n_out, T* __restrict__ out, int32_t* __restrict__ out_pos,
                 int32_t* __restrict__ out_span, int32_t* __restrict__ out_src_tok,
-                int8_t* __restrict__ out_src_sub, const int32_t* __restrict__ map) {
+                int8_t* __restrict__ out_src_sub, const int32_t* __restrict__ map,
+                unsigned int* status) {
   pdl_wait_then_trigger();
   const int lane = threadIdx.x & 31;
   const int64_t gwarp = (int64_t)blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
@@ -30,7 +31,7 @@ upsample_kernel(const T* __restrict__ latent, int B, int M, int gh, int gw, int 
   const int b = (int)(gwarp / M), i = (int)(gwarp % M);
   const int64_t in_tok = (int64_t)b * M + i;
   const UpsampleArgs<T> u{latent, M, gh, gw, C, n_out, pos_in, span_in, out,
-                          out_pos, out_span, out_src_tok, out_src_sub, map};
+                          out_pos, out_span, out_src_tok, out_src_sub, map, status};
   const GlobalRows<T> rows{latent, M, C * 4};
   upsample_token<T, kBilinear>(u, rows, b, i, tok_offset[in_tok], mask[in_tok] != 0, lane);
 }
@@ -58,7 +59,7 @@ cudaError_t launch_t(const void* latent, int B, int M, int gh, int gw, int C,
   e = launch_pdl(kern, dim3(grid), dim3(kWarpsPerCta * 32), 0, s,
                  static_cast<const T*>(latent), B, M, gh, gw, C, pos_in, span_in, mask,
                  tok_offset, n_out, static_cast<T*>(out), out_pos, out_span, out_src_tok,
-                 out_src_sub, static_cast<const int32_t*>(map));
+                 out_src_sub, static_cast<const int32_t*>(map), status);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

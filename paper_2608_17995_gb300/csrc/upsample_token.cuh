@@ -36,6 +36,7 @@ struct UpsampleArgs {
   // bilinear with a mixed input: the input frame's cell map [B,gh,gw]
   // (frame_map.cuh); NULL for a dense grid
   const int32_t* map = nullptr;
+  unsigned int* status = nullptr;  // device status word (an offset out of range)
 };
 
 // Where a token's C*4 source values are read from: element b's rows of the
@@ -75,6 +76,13 @@ __device__ __forceinline__ void upsample_token(const UpsampleArgs<T>& u, const S
     y = i / gw;
     x = i - y * gw;
     s = 1;
+  }
+  // the outputs must lie inside the element's sequence: an offset from the
+  // caller that does not is reported (AVITS_ERR_COVERAGE) and the token is
+  // not written
+  if (o < 0 || o > u.n_out - (sel ? 4 : 1)) {
+    if (lane == 0) raise_status(u.status, AVITS_ERR_COVERAGE);
+    return;
   }
   const T* src = rows.row(b, i);
   const int64_t out_tok0 = (int64_t)b * u.n_out + o;

@@ -632,6 +632,46 @@ def test_merge_detects_bad_tiling(av, orc, mode):
     assert np.array_equal(run(out, pos, span, 0), good)
 
 
+@pytest.mark.parametrize("mode", [0, 1])
+def test_upsample_reports_offsets_outside_the_sequence(av, orc, mode):
+    """avits_selective_upsample writes token i at the caller's tok_offset[i]
+    (Sec. 3.2 Stage 2).  An offset whose outputs would leave the sequence of
+    N_out = M + 3k tokens (a selected token starting 2 before the end, a
+    negative offset, a deferred token at N_out) raises AVITS_ERR_COVERAGE and
+    that token is not written; the other tokens are, and a consistent call
+    right after is clean and matches the oracle."""
+    import torch
+    lat = np.random.default_rng(1).standard_normal((1, 16, 8)).astype(np.float32)
+    mask = np.zeros((1, 16), np.uint8)
+    mask[0, [5, 10]] = 1
+    k = 2
+    off = (np.arange(16) + 3 * np.concatenate([[0], np.cumsum(mask[0])[:-1]])).astype(np.int32)[None]
+    NO = 16 + 3 * k
+    ref = orc.selective_upsample(lat, 4, 4, mask, mode="nearest" if mode == 0 else "bilinear")
+    bad = off.copy()
+    bad[0, 10] = NO - 2      # selected: its 4 children would end 2 past the sequence
+    bad[0, 3] = -1
+    bad[0, 15] = NO          # deferred: one past the end
+    out = torch.full((1, NO, 8), float("nan"), dtype=torch.float32, device="cuda")
+    pos = torch.full((1, NO, 2), -7, dtype=torch.int32, device="cuda")
+    span = torch.full((1, NO), -7, dtype=torch.int32, device="cuda")
+    st_ = torch.full((1, NO), -7, dtype=torch.int32, device="cuda")
+    ss = torch.full((1, NO), -7, dtype=torch.int8, device="cuda")
+    av.avits_selective_upsample(_dev(lat), 4, 4, _dev(mask), _dev(bad), k, out, pos, span, st_, ss,
+                                mode=mode)
+    assert _status(av) == 6
+    o, po = _np(out), _np(pos)
+    for i in range(16):      # every token with a valid offset is written as usual
+        if i in (3, 10, 15):
+            continue
+        n = 4 if mask[0, i] else 1
+        sl = slice(off[0, i], off[0, i] + n)
+        assert np.array_equal(o[0, sl], ref[0][0, sl]) and np.array_equal(po[0, sl], ref[1][0, sl])
+    got = _upsample(av, lat, "f32", 4, 4, mask, off, k, mode)
+    for a, b in zip(got, ref):
+        assert np.array_equal(a, b)
+
+
 # ------------------------------------------------------------ end to end ----
 
 @pytest.mark.parametrize("name,mode", [("tiny", "nearest"), ("flux1024", "nearest"),
