@@ -15,36 +15,41 @@
 // runs over all key tiles (128 keys), so O and the row statistics stay in
 // the CTA and no partial results cross CTAs (except Eq. 3's head sum).
 //
-// Tensor memory (512 columns): S_t of query tile t at columns [128t, 128t +
-// 128), O_t at [256 + Dt, 256 + D(t+1)).  P goes through shared memory, so
-// that S_t is free as soon as the softmax has loaded it: the next key tile's
-// S_t = Q_t K^T then runs on the tensor pipe while the softmax computes the
-// exponentials of this one.
+// Tensor memory (512 columns): one S buffer of 128 columns that the two query
+// tiles take in turn (S_0(g), S_1(g), S_0(g+1), ...), P_t as bf16 pairs (64
+// columns per tile), O_t (D columns per tile).  S is free as soon as its
+// softmax has loaded it, so the other tile's S runs on the tensor pipe while
+// this one's exponentials are computed; P never goes through shared memory
+// (the PV product reads it from tensor memory), which leaves shared memory
+// for Q, a 4-stage K / V ring and the O staging: per key tile and SM the
+// operand reads are 128 KB (S) + 64 KB (V), the copies 64 KB.
 //
 // Roles (12 warps):
 //   warp 0       TMA producer: Q tiles, then the K and V tiles through a
-//                3-stage ring in the order the MMAs consume them (K_0, K_1,
-//                V_0, K_2, V_1, ...), 128-byte swizzle.
+//                4-stage ring in the order the MMAs consume them (K_0, K_1,
+//                V_0, K_2, V_1, ...), 128-byte swizzle; a stage is refilled
+//                two key tiles after its last use.
 //   warps 1, 2   MMA issuers of query tile 0 / 1 (warp 1 owns tensor
-//                memory): for key tile g, S_t(g) = Q_t K_g^T once the softmax
-//                has loaded S_t(g-1), then O_t += P_t(g-1) V_(g-1) once that P
-//                is in shared memory.  Both products are tcgen05.mma kind::f16
-//                from shared memory; V is read in its natural [keys, d] layout
-//                as an MN-major operand (no transpose copy).
+//                memory): for key tile g, S_t(g) = Q_t K_g^T (from shared
+//                memory) once the S before it has been loaded, then O_t +=
+//                P_t(g-1) V_(g-1) (A = P_t from tensor memory, the
+//                tcgen05.mma TS form; V read in its natural [keys, d] layout
+//                as an MN-major shared-memory operand, no transpose copy) once
+//                that P has been written.
 //   warp 3       no role.
 //   warps 4-7    softmax and epilogue of query tile 0, warps 8-11 of tile 1:
-//                one row per thread (TMEM lane); the row's 128 S columns are loaded into registers and
-//                S_t released; the row maximum; the running maximum is raised
-//                only when a key tile's maximum exceeds it by more than 2^8
-//                (P <= 256 otherwise, no loss in bf16 or the fp32
-//                accumulator), and then l and O are rescaled (O in tensor
-//                memory, by the whole warp); the exponentials (packed FMA +
-//                MUFU), the fp32 sums over all keys and over the text keys
-//                (the only addition the score needs) and the bf16 P row, written
-//                to shared memory in the K-major 128-byte-swizzled layout the
-//                MMA reads.  The epilogue divides O by the row sum, stages it
-//                in the P buffer and stores it with one bulk tensor copy per 64
-//                columns.
+//                one row per thread (TMEM lane); the row's 128 S columns are
+//                loaded into registers and the S buffer released; the row
+//                maximum; the running maximum is raised only when a key
+//                tile's maximum exceeds it by more than 2^8 (P <= 256
+//                otherwise, no loss in bf16 or the fp32 accumulator), and then
+//                l and O are rescaled (O in tensor memory, by the whole warp);
+//                the exponentials (packed FMA + MUFU), the fp32 sums over all
+//                keys and over the text keys (the only addition the score
+//                needs) and the bf16 P row, written to tensor memory once the
+//                previous PV product has read P_t.  The epilogue divides O by
+//                the row sum and stores it 64 columns at a time through a
+//                swizzled staging block with a bulk tensor copy.
 // Every wait is bounded (avits_common.cuh); after a timeout every role skips
 // its remaining work, drains what it issued and the CTA releases tensor
 // memory and exits.
@@ -72,16 +77,19 @@ template <int D>
 struct Cfg {
   static constexpr int kCB = D / 64;                   // 128-byte column blocks per row
   static constexpr int kTileBytes = kCB * kBM * 128;   // one 128-row bf16 tile
-  static constexpr int kStages = (D == 128) ? 3 : 6;   // K / V ring
+  static constexpr int kStages = (D == 128) ? 4 : 8;   // K / V ring
   static constexpr int kQBytes = kQTiles * kTileBytes;
   static constexpr int kKVBytes = kStages * kTileBytes;
   static constexpr uint32_t kIdescPV = idesc_bf16(kBM, D, true);
 };
-// P of one query tile: 128 rows x 128 keys bf16 (two 128-byte column blocks);
-// at a unit's end the same buffer stages that tile's O (D <= 128 columns)
-constexpr int kPTileBytes = 2 * kBM * 128;
-constexpr int kPBytes = kQTiles * kPTileBytes;
-constexpr int kMaxStages = 6;
+// O staging at a unit's end: per query tile one 128-row x 64-column bf16
+// block (128-byte swizzle), stored with a bulk tensor copy per 64 columns
+constexpr int kStageTileBytes = kBM * 128;
+constexpr int kStageBytes = kQTiles * kStageTileBytes;
+constexpr int kMaxStages = 8;
+// Tensor memory columns: the S buffer both query tiles share, then P_t (bf16
+// pairs, 64 columns per tile), then O_t (D columns per tile).
+constexpr int kColS = 0, kColP = kBN, kColO = kBN + kQTiles * (kBN / 2);
 
 struct Bars {
   uint64_t q_full[kQTiles], q_empty[kQTiles];
@@ -94,7 +102,7 @@ struct Bars {
 
 template <int D>
 constexpr int smem_bytes() {
-  return Cfg<D>::kQBytes + Cfg<D>::kKVBytes + kPBytes + (int)sizeof(Bars) + 1024;
+  return Cfg<D>::kQBytes + Cfg<D>::kKVBytes + kStageBytes + (int)sizeof(Bars) + 1024;
 }
 
 struct AttnParams {
@@ -164,10 +172,11 @@ __device__ __forceinline__ void rescale_o(uint32_t tO, float f) {
 }
 
 // Exponentials of 32 S columns (first key col0) against the running maximum
-// m, in place (r then holds the fp32 softmax numerators), and their fp32 sums
-// over all keys and over the text keys.  kKind: 0 = valid image keys, 1 =
-// valid text keys, 2 = general (keys beyond Nk give 0, text keys counted one
-// by one).
+// m, their fp32 sums over all keys and over the text keys, and the bf16
+// numerators packed in place: r[i] (i < 16) = keys 2i, 2i + 1 (the even key in
+// the low half), the layout the PV product reads P_t in from tensor memory.
+// kKind: 0 = valid image keys, 1 = valid text keys, 2 = general (keys beyond
+// Nk give 0, text keys counted one by one).
 template <int kKind>
 __device__ __forceinline__ void exp_chunk(uint32_t (&r)[32], int col0, int Nk, int L, float c,
                                           float m, float& la, float& lt) {
@@ -185,8 +194,7 @@ __device__ __forceinline__ void exp_chunk(uint32_t (&r)[32], int col0, int Nk, i
       if (col0 + e + 1 < L) t0 += e1;
     }
     fadd2(s0, s1, e0, e1);
-    r[e] = __float_as_uint(e0);
-    r[e + 1] = __float_as_uint(e1);
+    r[e >> 1] = pack_bf16x2(e0, e1);   // slot e / 2 <= e has been read
   }
   const float cs = s0 + s1;
   la += cs;
@@ -204,18 +212,14 @@ __device__ __forceinline__ void exp_tile(uint32_t (&r0)[32], uint32_t (&r1)[32],
   exp_chunk<kKind>(r3, key0 + 96, Nk, L, c, m, la, lt);
 }
 
-// 32 fp32 numerators -> bf16, four 16-byte chunks of the row's P block: chunk
-// q at position (jj0 + q) ^ (row & 7) of the 128-byte row (the K-major
-// 128-byte swizzle the MMA reads).
-__device__ __forceinline__ void store_p(const uint32_t (&r)[32], uint8_t* rowp, int jj0, int rsw) {
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    *reinterpret_cast<uint4*>(rowp + (((jj0 + q) ^ rsw) << 4)) =
-        make_uint4(pack_bf16x2(__uint_as_float(r[8 * q]), __uint_as_float(r[8 * q + 1])),
-                   pack_bf16x2(__uint_as_float(r[8 * q + 2]), __uint_as_float(r[8 * q + 3])),
-                   pack_bf16x2(__uint_as_float(r[8 * q + 4]), __uint_as_float(r[8 * q + 5])),
-                   pack_bf16x2(__uint_as_float(r[8 * q + 6]), __uint_as_float(r[8 * q + 7])));
-  }
+// The 16 packed words at the front of r (32 keys of P) into 16 tensor-memory
+// columns of this thread's lane.
+__device__ __forceinline__ void tmem_st_p(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+      AVITS_I8(0), AVITS_I8(8)
+      : "memory");
 }
 
 struct RowState {
@@ -240,8 +244,8 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sQ = smem;
   uint8_t* sKV = sQ + C::kQBytes;
-  uint8_t* sP = sKV + C::kKVBytes;   // P of each query tile; the O staging at a unit's end
-  Bars* bars = reinterpret_cast<Bars*>(sP + kPBytes);
+  uint8_t* sStage = sKV + C::kKVBytes;   // O staging, one 64-column block per tile
+  Bars* bars = reinterpret_cast<Bars*>(sStage + kStageBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n_my = (p.n_units - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
@@ -350,19 +354,21 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
     }
   } else if (warp == 1 || warp == 2) {
     // -------------------------------------------------------- MMA issuers --
-    // Key tile g: S_t(g) = Q_t K_g^T as soon as the softmax has loaded
-    // S_t(g-1); then O_t += P_t(g-1) V_(g-1) once P_t(g-1) is in shared
-    // memory.  The tensor pipe so holds the next S while the softmax works.
+    // Key tile g: S_t(g) = Q_t K_g^T into the S buffer both tiles share, as
+    // soon as the other tile's softmax has loaded the S before it (S_0(g)
+    // after S_1(g-1), S_1(g) after S_0(g)); then O_t += P_t(g-1) V_(g-1) with
+    // P_t from tensor memory once the softmax has written it.  The next S so
+    // runs on the tensor pipe while the softmax works on this one.
     const int t = warp - 1;
     if (lane == 0) {
       bool ok = true;
       const uint32_t q_lo = sw128_desc_lo(sQ + t * C::kTileBytes);
-      const uint32_t p_lo = sw128_desc_lo(sP + t * kPTileBytes);
       const uint32_t kv_lo0 = sw128_desc_lo(sKV);
       const uint32_t v_lo0 = sw128_mn_desc_lo(sKV, kBM * 128);
       const uint32_t d_hi = sw128_desc_hi();
-      const uint32_t tS = tmem + (uint32_t)(t * kBN);
-      const uint32_t tO = tmem + (uint32_t)(2 * kBN + t * D);
+      const uint32_t tS = tmem + (uint32_t)kColS;
+      const uint32_t tP = tmem + (uint32_t)(kColP + t * (kBN / 2));
+      const uint32_t tO = tmem + (uint32_t)(kColO + t * D);
       for (int gi = 0; gi <= G && ok; ++gi) {
         if (gi < G) {
           const int ui = gi / p.n_kt, j = gi - ui * p.n_kt;
@@ -370,8 +376,12 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
           ok = mbar_wait_bounded(&bars->kv_full[sk], (uint32_t)((lk / C::kStages) & 1), abort_flag, p.status);
           if (ok && j == 0)
             ok = mbar_wait_bounded(&bars->q_full[t], (uint32_t)(ui & 1), abort_flag, p.status);
-          if (ok && gi > 0)   // the softmax has loaded S_t(gi - 1)
-            ok = mbar_wait_bounded(&bars->s_empty[t], (uint32_t)((gi - 1) & 1), abort_flag, p.status);
+          // the shared S buffer: the previous S in the order S_0(0), S_1(0),
+          // S_0(1), ... has been loaded by its softmax
+          if (ok && t == 0 && gi > 0)
+            ok = mbar_wait_bounded(&bars->s_empty[1], (uint32_t)((gi - 1) & 1), abort_flag, p.status);
+          if (ok && t == 1)
+            ok = mbar_wait_bounded(&bars->s_empty[0], (uint32_t)(gi & 1), abort_flag, p.status);
           if (!ok) break;
           fence_after();
           const uint32_t k_lo = kv_lo0 + (uint32_t)((sk * C::kTileBytes) >> 4);
@@ -397,11 +407,9 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
           fence_after();
           const uint32_t v_lo = v_lo0 + (uint32_t)((sv * C::kTileBytes) >> 4);
 #pragma unroll
-          for (int kk = 0; kk < kBN / 16; ++kk) {   // 16 keys: 16 P columns, 16 V rows
-            const uint32_t off = (uint32_t)(((kk >> 2) * (kBM * 128) + (kk & 3) * 32) >> 4);
-            mma_ss(tO, p_lo + off, v_lo + (uint32_t)((kk * 16 * 128) >> 4), d_hi, C::kIdescPV,
-                   (jg > 0 || kk > 0) ? 1u : 0u);
-          }
+          for (int kk = 0; kk < kBN / 16; ++kk)   // 16 keys: 8 P columns, 16 V rows
+            mma_ts(tO, tP + (uint32_t)(kk * 8), v_lo + (uint32_t)((kk * 16 * 128) >> 4), d_hi,
+                   C::kIdescPV, (jg > 0 || kk > 0) ? 1u : 0u);
           mma_commit(&bars->pv_done[t]);
           mma_commit(&bars->kv_empty[sv]);
           if (jg == p.n_kt - 1) mma_commit(&bars->o_full[t]);
@@ -416,12 +424,16 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
     const int t = (warp - 4) >> 2;
     const int quad = warp & 3;             // TMEM lane quadrant this warp may access
     const int rowt = quad * 32 + lane;     // row within the tile = TMEM lane
-    const int bar_id = 1 + t;              // named barrier of the tile's 128 threads
     const bool leader = (quad == 0 && lane == 0);
+    // named barrier of the tile's 128 threads: 1 + t (literal ids, so that
+    // the kernel reserves only the barriers it uses)
+    auto tile_sync = [&]() { if (t == 0) bar_sync(1, 128); else bar_sync(2, 128); };
+    auto tile_and = [&](bool v) { return t == 0 ? bar_and(1, 128, v) : bar_and(2, 128, v); };
     const uint32_t lane_off = (uint32_t)(quad * 32) << 16;
-    const uint32_t tS = tmem + lane_off + (uint32_t)(t * kBN);
-    const uint32_t tO = tmem + lane_off + (uint32_t)(2 * kBN + t * D);
-    uint8_t* sPt = sP + t * kPTileBytes;
+    const uint32_t tS = tmem + lane_off + (uint32_t)kColS;
+    const uint32_t tP = tmem + lane_off + (uint32_t)(kColP + t * (kBN / 2));
+    const uint32_t tO = tmem + lane_off + (uint32_t)(kColO + t * D);
+    uint8_t* sSt = sStage + t * kStageTileBytes;
     const float c = p.c_log2;
     bool ok = true;
     int gi = 0;
@@ -435,8 +447,8 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
         ok = __all_sync(0xffffffffu, ok);   // tcgen05.ld / st are warp-collective
         if (ok) {
           fence_after();
-          // the row's 128 S columns into registers; S_t is then free for the
-          // next key tile's MMA
+          // the row's 128 S columns into registers; the S buffer is then free
+          // for the other tile's S
           uint32_t r0[32], r1[32], r2[32], r3[32];
           tmem_ld32(tS, r0);
           tmem_ld32(tS + 32, r1);
@@ -467,8 +479,8 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
             st.lt *= f;
             st.m = mt;
           }
-          // the numerators in place while the previous PV product may still
-          // be reading the P buffer; the kind is uniform over the warp
+          // the numerators (bf16 pairs) while the previous PV product may
+          // still be reading P_t; the kind is uniform over the warp
           if (key0 + kBN <= p.Nk && key0 >= p.L)
             exp_tile<0>(r0, r1, r2, r3, key0, p.Nk, p.L, c, st.m, st.la, st.lt);
           else if (key0 + kBN <= p.Nk && key0 + kBN <= p.L)
@@ -481,56 +493,63 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
             ok = __all_sync(0xffffffffu, w);
           }
           if (ok) {
-            uint8_t* rowp0 = sPt + rowt * 128;
-            uint8_t* rowp1 = rowp0 + kBM * 128;
-            const int rsw = rowt & 7;
-            store_p(r0, rowp0, 0, rsw);
-            store_p(r1, rowp0, 4, rsw);
-            store_p(r2, rowp1, 0, rsw);
-            store_p(r3, rowp1, 4, rsw);
+            // P_t into tensor memory: column c of the row holds keys 2c, 2c + 1
+            tmem_st_p(tP, r0);
+            tmem_st_p(tP + 16, r1);
+            tmem_st_p(tP + 32, r2);
+            tmem_st_p(tP + 48, r3);
             // the warp rescales its O rows together when any of them moved
             // (f = 1 leaves a row unchanged)
-            if (j > 0 && __any_sync(0xffffffffu, up)) {
-              rescale_o<D>(tO, f);
-              tmem_wait_st();
-            }
-            fence_async_shared();   // P is read by the tensor core (async proxy)
+            if (j > 0 && __any_sync(0xffffffffu, up)) rescale_o<D>(tO, f);
+            tmem_wait_st();
             fence_before();
           }
         }
         __syncwarp();
         if (ok && lane == 0) mbar_arrive(&bars->p_full[t]);
       }
-      // ---- epilogue: O / l -> bf16 -> swizzled staging (the P buffer, free
-      // once the last PV product completed) -> TMA store
+      // ---- epilogue: O / l -> bf16 -> swizzled staging, 64 columns at a
+      // time -> TMA store
       ok = ok && (*abort_flag == 0) &&
            mbar_wait_bounded(&bars->o_full[t], (uint32_t)(ui & 1), abort_flag, p.status);
       ok = __all_sync(0xffffffffu, ok);
-      if (ok) {
-        fence_after();
-        const float inv = 1.f / st.la;
+      const float inv = 1.f / st.la;
+      const int row0 = qp * kUnitRows + t * kBM;
 #pragma unroll 1
-        for (int k = 0; k < D / 32; ++k) {
-          uint32_t r[32];
-          tmem_ld32(tO + 32 * k, r);
-          tmem_wait32(r);
-          uint32_t w[16];
+      for (int cb = 0; cb < C::kCB; ++cb) {
+        if (ok) {
+          fence_after();
+#pragma unroll 1
+          for (int k = 0; k < 2; ++k) {
+            uint32_t r[32];
+            tmem_ld32(tO + 64 * cb + 32 * k, r);
+            tmem_wait32(r);
+            uint32_t w[16];
 #pragma unroll
-          for (int e = 0; e < 16; ++e)
-            w[e] = pack_bf16x2(__uint_as_float(r[2 * e]) * inv, __uint_as_float(r[2 * e + 1]) * inv);
-          const int cb = (32 * k) >> 6;
-          const int jj0 = ((32 * k) & 63) >> 3;
-          uint8_t* rowp = sPt + cb * (kBM * 128) + rowt * 128;
+            for (int e = 0; e < 16; ++e)
+              w[e] = pack_bf16x2(__uint_as_float(r[2 * e]) * inv, __uint_as_float(r[2 * e + 1]) * inv);
+            uint8_t* rowp = sSt + rowt * 128;
 #pragma unroll
-          for (int q = 0; q < 4; ++q)
-            *reinterpret_cast<uint4*>(rowp + (((jj0 + q) ^ (rowt & 7)) << 4)) =
-                make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+            for (int q = 0; q < 4; ++q)
+              *reinterpret_cast<uint4*>(rowp + (((4 * k + q) ^ (rowt & 7)) << 4)) =
+                  make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+          }
+          fence_before();
         }
-        fence_before();
+        if (cb == C::kCB - 1) {   // every O column of this unit has been read
+          __syncwarp();
+          if (ok && lane == 0) mbar_arrive(&bars->o_empty[t]);
+        }
+        fence_async_shared();
+        const bool all_ok = tile_and(ok);
+        if (all_ok && leader && row0 < p.Mq) {   // a tile past the end stores nothing
+          tma_store_4d(&tmO, sSt, cb * 64, row0, h, b);
+          bulk_commit();
+          bulk_wait_read();   // the staging is rewritten by the next block
+        }
+        tile_sync();
       }
-      __syncwarp();
-      if (ok && lane == 0) mbar_arrive(&bars->o_empty[t]);
-      const int row = qp * kUnitRows + t * kBM + rowt;
+      const int row = row0 + rowt;
       if (ok && row < p.Mq) {
         const float ln2 = 0.69314718055994530942f;
         if (p.lse) {
@@ -542,15 +561,6 @@ attention_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_consta
           head_sum_add(p.acc + (long long)b * p.rows_pad + row, p.H, st.lt / st.la, p.weight,
                        p.accumulate, p.A + (long long)b * p.Mq + row);
       }
-      fence_async_shared();
-      const bool all_ok = bar_and(bar_id, 128, ok);
-      if (all_ok && leader && qp * kUnitRows + t * kBM < p.Mq) {   // a tile past the end stores nothing
-        for (int cb = 0; cb < C::kCB; ++cb)
-          tma_store_4d(&tmO, sPt + cb * (kBM * 128), cb * 64, qp * kUnitRows + t * kBM, h, b);
-        bulk_commit();
-        bulk_wait_read();   // the staging is the next unit's P buffer
-      }
-      bar_sync(bar_id, 128);
     }
     if (leader) bulk_wait_all();
   }
