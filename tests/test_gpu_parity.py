@@ -240,6 +240,8 @@ def test_spatial_bf16_configs(av, orc, name, nrows):
     (3, 2, 64, 1, 5, 128),       # one text key
     (1, 2, 129, 0, 7, 64),       # no text: mass 0
     (1, 2, 40, 60, 0, 128),      # Nk < 128
+    (2, 3, 400, 77, 45, 128),    # CTA pairs (two row units per head), ragged second unit
+    (1, 5, 1000, 256, 3, 128),   # CTA pairs, 4 row units per head, odd head count
 ])
 def test_spatial_tc_ragged_shapes(av, orc, B, H, M, L, R, d):
     from paper_2608_17995_gb300.workloads import to_bf16_bits
