@@ -583,7 +583,7 @@ def config_measure(torch, av, dev, stream, peaks, name, nsets=3):
     """Another configuration's transition: the whole step and the spatial
     call, inputs rotated over nsets copies (> L2).  FLUX-2048 (M = 4096,
     Nk = 4608, 116 GFLOP in the spatial score): every CTA of the spatial
-    kernel runs ~90 items, so start-up and the finalize are a small share of
+    kernel runs ~90 items, so start-up and the merge are a small share of
     its time.  Editing (M = 1024 with 4096 reference keys, Nk = 5632)."""
     from paper_2608_17995_gb300.pipeline import TransitionBuffers
     from paper_2608_17995_gb300.workloads import make_transition
